@@ -1,0 +1,88 @@
+"""Closed-form cost model of the Pr^2 layer (host logic, no GPU).
+
+* Table 4 / App. E.2 of the paper: index cache 4*T*L*k bytes (int32 indices), feature cache
+  T_c*L*(2d + 4N) bytes (bf16 hidden features + fp32 router logits), predictor FLOPs 2*L*d*N per
+  token, and the FFN ratio 2*L*d*N / (6*L*(k+s)*d*m).
+* Algorithmic bytes and FLOPs per kernel of this library, used as the roofline numerators.  They
+  count each tensor a kernel must touch exactly once (compulsory traffic), nothing else.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+
+def index_cache_bytes(T: int, L: int, k: int) -> int:
+    """Int32 replay indices for one response of T tokens over L layers (Table 4, App. E.2)."""
+    return 4 * T * L * k
+
+
+def feature_cache_bytes(T_c: int, L: int, d: int, N: int) -> int:
+    """bf16 h_old [d] + fp32 p_old [N] for T_c retained positions over L layers (Table 4)."""
+    return T_c * L * (2 * d + 4 * N)
+
+
+def predictor_flops_per_token(L: int, d: int, N: int) -> int:
+    """Extra route-recording FLOPs of the L predictor projections h W_p (App. E.2)."""
+    return 2 * L * d * N
+
+
+def ffn_ratio(L: int, d: int, N: int, k: int, s: int, m: int) -> float:
+    """Predictor FLOPs over the active gated-MLP FLOPs 6*L*(k+s)*d*m per token (App. E.2)."""
+    return predictor_flops_per_token(L, d, N) / (6 * L * (k + s) * d * m)
+
+
+@dataclass(frozen=True)
+class KernelWork:
+    """Algorithmic work of one launch: bytes that must cross HBM and FLOPs that must be done."""
+
+    bytes: int
+    flops: int
+
+
+def _esz(dtype: str) -> int:
+    return 4 if dtype == "fp32" else 2
+
+
+def route_predict_work(T: int, d: int, N: int, k: int, dtype: str = "bf16",
+                       write_logits: bool = True) -> KernelWork:
+    """Read h [T,d] and [W; W_p] [2N,d]; write idx + gates [T,k] (+ p_old [T,N] fp32)."""
+    e = _esz(dtype)
+    b = T * d * e + 2 * N * d * e + T * k * 8 + (T * N * 4 if write_logits else 0)
+    return KernelWork(b, 2 * T * d * 2 * N)
+
+
+def route_replay_work(T: int, d: int, N: int, k: int, dtype: str = "bf16",
+                      write_probs: bool = False) -> KernelWork:
+    """Read h, W [N,d] and idx [T,k]; write gates [T,k] (+ rho [T,N] fp32)."""
+    e = _esz(dtype)
+    b = T * d * e + N * d * e + T * k * 4 + T * k * 4 + (T * N * 4 if write_probs else 0)
+    return KernelWork(b, 2 * T * d * N)
+
+
+def dispatch_work(T: int, d: int, k: int, dtype: str = "bf16") -> KernelWork:
+    """Histogram + scan + stable rank + row gather: read idx and h once, write perm, inv and the
+    permuted rows X_perm [T*k, d]."""
+    e = _esz(dtype)
+    return KernelWork(T * k * 4 + T * d * e + 2 * T * k * 4 + T * k * d * e, 0)
+
+
+def expert_gate_up_work(rows: int, d: int, m: int, experts_hit: int,
+                        dtype: str = "bf16") -> KernelWork:
+    """Grouped [X_e] x [W_gate; W_up]_e^T with the SwiGLU epilogue: read X_perm and the gate/up
+    weights of every expert hit, write H [rows, m]."""
+    e = _esz(dtype)
+    return KernelWork(rows * d * e + experts_hit * 2 * m * d * e + rows * m * e,
+                      2 * rows * d * 2 * m)
+
+
+def expert_down_work(rows: int, d: int, m: int, experts_hit: int,
+                     dtype: str = "bf16") -> KernelWork:
+    """Grouped H_e x W_down,e^T: read H and the down weights of every expert hit, write Y."""
+    e = _esz(dtype)
+    return KernelWork(rows * m * e + experts_hit * d * m * e + rows * d * e, 2 * rows * m * d)
+
+
+def combine_work(T: int, d: int, k: int, n_shared: int = 0, dtype: str = "bf16") -> KernelWork:
+    """out[t] = sum_s g[t,s] Y[inv[t,s]] (+ shared rows): read Y, gates, inv; write out."""
+    e = _esz(dtype)
+    return KernelWork(T * k * d * e + T * k * 8 + T * n_shared * d * e + T * d * e, 0)

@@ -1,0 +1,34 @@
+"""The closed-form cost model against the values Table 4 (App. E.2) prints."""
+import json
+import os
+
+import pytest
+
+from paper_2606_00395_gb300 import cost
+
+GOLDEN = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "table4_overheads.json")))
+
+
+def _printed(x, ref):
+    """x rounded the way the table prints ref (same number of decimals)."""
+    s = repr(ref)
+    dec = len(s.split(".")[1]) if "." in s else 0
+    return round(x, dec) == ref
+
+
+@pytest.mark.parametrize("row", GOLDEN["rows"], ids=[r["model"] for r in GOLDEN["rows"]])
+def test_table4_closed_forms(row):
+    L, d, N, k, s, m, T, Tc = (row[x] for x in ("L", "d", "N", "k", "s", "m", "T", "T_c"))
+    assert _printed(cost.index_cache_bytes(T, L, k) / 1e6, row["index_cache_MB"])
+    assert _printed(cost.feature_cache_bytes(Tc, L, d, N) / 1e6, row["feature_cache_MB"])
+    assert _printed(cost.predictor_flops_per_token(L, d, N) / 1e6, row["flops_M"])
+    assert _printed(100 * cost.ffn_ratio(L, d, N, k, s, m), row["ffn_ratio_pct"])
+
+
+def test_kernel_work_counts_each_tensor_once():
+    w = cost.route_predict_work(4096, 2048, 128, 8)
+    assert w.bytes == 4096 * 2048 * 2 + 256 * 2048 * 2 + 4096 * 8 * 8 + 4096 * 128 * 4
+    assert w.flops == 2 * 4096 * 2048 * 256
+    g = cost.expert_gate_up_work(32768, 2048, 768, 128)
+    dn = cost.expert_down_work(32768, 2048, 768, 128)
+    assert g.flops + dn.flops == 6 * 4096 * 8 * 2048 * 768

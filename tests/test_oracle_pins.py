@@ -1,0 +1,297 @@
+"""Pins for the CPU oracle: each check compares it with something other than itself.
+
+The paper prints no worked numeric example of the layer, so the pins are closed forms, special
+cases that reduce to a textbook or library routine, brute force on tiny inputs, and the
+inequalities of App. B (Lemma topk_regret, Pinsker).  ``test_oracle_mutants.py`` plants
+plausible mistakes in copies of the oracle and checks that these pins catch each one.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_00395_gb300 import synth
+
+
+def _rand(shape, seed, scale=1.0):
+    g = torch.Generator().manual_seed(seed)
+    return (torch.randn(*shape, generator=g) * scale).contiguous()
+
+
+def _f64(t):
+    return t.double().numpy()
+
+
+# ------------------------------------------------------------------ routing (Sec. 4.1)
+
+def test_softmax_rows_sum_to_one():
+    h, W, Wp = _rand((64, 32), 1), _rand((16, 32), 2, 0.3), _rand((16, 32), 3, 0.3)
+    r = oracle.route_predict(h, W, Wp, 4)
+    assert np.all(np.abs(r["probs"].sum(1) - 1.0) < 1e-12)
+    assert np.all(r["probs"] > 0)
+
+
+def test_selector_rows_give_closed_form_logits_and_softmax():
+    """W rows are basis vectors: p_e = h[pi(e)] exactly, so rho-hat has a closed form.
+
+    A transposed weight read, a wrong row index, or a dropped predictor term changes these."""
+    T, d, N, k = 8, 12, 5, 2
+    pi = [7, 0, 11, 3, 5]
+    h = _rand((T, d), 4)
+    W = torch.zeros(N, d)
+    for e, i in enumerate(pi):
+        W[e, i] = 1.0
+    Wp = torch.zeros(N, d)
+    Wp[2, 1] = 0.5  # b_2 = 0.5 * h[:, 1]
+    r = oracle.route_predict(h, W, Wp, k)
+    hd = _f64(h)
+    logits = np.stack([hd[:, i] for i in pi], 1)
+    assert np.array_equal(r["logits"], logits)
+    for t in range(T):
+        z = [hd[t, pi[e]] + (0.5 * hd[t, 1] if e == 2 else 0.0) for e in range(N)]
+        den = sum(math.exp(v) for v in z)
+        for e in range(N):
+            assert abs(r["probs"][t, e] - math.exp(z[e]) / den) < 1e-14
+
+
+def test_two_experts_is_a_sigmoid_of_the_logit_gap():
+    h, W, Wp = _rand((32, 8), 5), _rand((2, 8), 6, 0.5), _rand((2, 8), 7, 0.5)
+    r = oracle.route_predict(h, W, Wp, 1)
+    z = _f64(h) @ _f64(W).T + _f64(h) @ _f64(Wp).T
+    sig = 1.0 / (1.0 + np.exp(z[:, 1] - z[:, 0]))
+    assert np.max(np.abs(r["probs"][:, 0] - sig)) < 1e-14
+
+
+@pytest.mark.parametrize("N", [1, 2, 5, 16])
+def test_topk_equals_brute_force_sort(N):
+    T, d = 48, 6
+    h, W, Wp = _rand((T, d), 10 + N), _rand((N, d), 20 + N), _rand((N, d), 30 + N, 0.2)
+    for k in range(1, N + 1):
+        r = oracle.route_predict(h, W, Wp, k)
+        for t in range(T):
+            order = sorted(range(N), key=lambda e: (-r["probs"][t, e], e))
+            assert list(r["idx"][t]) == order[:k]
+            assert np.array_equal(r["gates"][t], r["probs"][t, order[:k]])
+            want = r["probs"][t, order[k - 1]] - r["probs"][t, order[k]] if k < N else math.inf
+            assert r["margin"][t] == want
+
+
+def test_uniform_router_breaks_ties_to_lower_index():
+    """W = W_p = 0 gives rho-hat = 1/N; W_p = -W cancels the router exactly (sign of b)."""
+    T, d, N, k = 6, 10, 7, 3
+    h = _rand((T, d), 40)
+    W = _rand((N, d), 41)
+    for Wr, Wq in ((torch.zeros(N, d), torch.zeros(N, d)), (W, -W)):
+        r = oracle.route_predict(h, Wr, Wq, k)
+        assert np.array_equal(r["idx"], np.tile(np.arange(k, dtype=np.int32), (T, 1)))
+        assert np.all(r["gates"] == 1.0 / N)
+        assert np.all(r["margin"] == 0.0)
+
+
+def test_zero_predictor_is_plain_topk_routing():
+    """W_p = 0 reduces Pr^2 rollout routing to the router's own top-k (routing replay, R2)."""
+    T, d, N, k = 40, 16, 12, 3
+    h, W = _rand((T, d), 50), _rand((N, d), 51, 0.4)
+    r = oracle.route_predict(h, W, torch.zeros(N, d), k)
+    p = _f64(h) @ _f64(W).T
+    ref = np.argsort(-p, axis=1, kind="stable")[:, :k]
+    assert np.array_equal(r["idx"], ref)
+    rep = oracle.route_replay(h, W, r["idx"])
+    assert np.array_equal(rep["gates"], r["gates"]) and rep["bad"] == 0
+
+
+def test_predictor_alone_routes_by_its_own_projection():
+    """W = 0: the route is the top-k of h W_p (the predictor term is present and added)."""
+    T, d, N, k = 40, 16, 12, 3
+    h, Wp = _rand((T, d), 52), _rand((N, d), 53, 0.4)
+    r = oracle.route_predict(h, torch.zeros(N, d), Wp, k)
+    b = _f64(h) @ _f64(Wp).T
+    assert np.array_equal(r["idx"], np.argsort(-b, axis=1, kind="stable")[:, :k])
+    assert np.all(r["logits"] == 0.0)  # p_old excludes the predictor bias
+
+
+def test_replay_gates_gather_current_router_probabilities():
+    T, d, N, k = 30, 16, 10, 4
+    h, W = _rand((T, d), 60), _rand((N, d), 61, 0.4)
+    idx = np.stack([np.random.default_rng(t).permutation(N)[:k] for t in range(T)]).astype(np.int32)
+    rep = oracle.route_replay(h, W, idx)
+    p = _f64(h) @ _f64(W).T
+    ref = np.exp(p - p.max(1, keepdims=True))
+    ref /= ref.sum(1, keepdims=True)
+    assert np.max(np.abs(rep["probs"] - ref)) < 1e-14
+    assert np.array_equal(rep["gates"], np.take_along_axis(rep["probs"], idx, 1))
+
+
+def test_replay_flags_invalid_and_duplicate_indices():
+    T, d, N = 4, 8, 6
+    h, W = _rand((T, d), 62), _rand((N, d), 63)
+    idx = np.array([[0, 1], [6, 2], [-1, 3], [4, 4]], np.int32)
+    rep = oracle.route_replay(h, W, idx)
+    assert rep["bad"] == 3
+    assert rep["gates"][1, 0] == 0 and rep["gates"][2, 0] == 0 and rep["gates"][3, 1] == 0
+    assert rep["gates"][3, 0] == rep["probs"][3, 4]
+
+
+def _kl(p, q):
+    return float(np.sum(p * (np.log(p) - np.log(q))))
+
+
+def test_lemma_topk_regret_and_margin_condition():
+    """App. B, Lemma topk_regret: p(S*) - p(S_hat) <= sqrt(2 KL(p||p_hat)); if
+    KL < Delta_k(p)^2 / 2 the supports coincide; Pinsker: ||p - p_hat||_inf <= sqrt(KL/2)."""
+    T, d, N, k = 400, 24, 16, 4
+    h = _rand((T, d), 70)
+    W = _rand((N, d), 71, 0.5)
+    hits = 0
+    for trial, scale in enumerate((0.002, 0.02, 0.1, 0.5)):
+        Wp = _rand((N, d), 72 + trial, scale)
+        pred = oracle.route_predict(h, W, Wp, k)                     # rho-hat = Softmax(p + b)
+        cur = oracle.route_predict(h, W, torch.zeros(N, d), k)       # rho = Softmax(p), TopK
+        for t in range(T):
+            p, q = cur["probs"][t], pred["probs"][t]
+            kl = _kl(p, q)
+            s_star, s_hat = cur["idx"][t], pred["idx"][t]
+            assert p[s_star].sum() - p[s_hat].sum() <= math.sqrt(2 * kl) + 1e-15
+            assert np.max(np.abs(p - q)) <= math.sqrt(kl / 2) + 1e-15
+            if kl < cur["margin"][t] ** 2 / 2:
+                hits += 1
+                assert set(s_star) == set(s_hat)
+    assert hits > 100  # the margin branch is exercised
+
+
+# ------------------------------------------------------------------ dispatch
+
+@pytest.mark.parametrize("T,k,N", [(1, 1, 1), (37, 3, 5), (64, 8, 16), (0, 2, 4)])
+def test_permute_is_a_stable_counting_sort(T, k, N):
+    rng = np.random.default_rng(T * 100 + k)
+    idx = np.array([rng.permutation(N)[:k] for _ in range(T)], np.int32).reshape(T, k)
+    r = oracle.permute(idx, N)
+    flat = idx.reshape(-1)
+    assert np.array_equal(r["counts"], np.bincount(flat, minlength=N))
+    assert r["counts"].sum() == T * k and r["offsets"][N] == T * k
+    assert list(r["perm"]) == sorted(range(T * k), key=lambda f: (flat[f], f))
+    assert np.array_equal(r["inv"][r["perm"]], np.arange(T * k))
+
+
+def test_permute_skips_invalid_slots():
+    idx = np.array([[1, 1], [0, 9], [2, -3]], np.int32)
+    r = oracle.permute(idx, 3)
+    assert r["bad"] == 3 and list(r["counts"]) == [1, 1, 1]
+    assert list(r["perm"]) == [2, 0, 4] and list(r["inv"]) == [1, -1, 0, -1, 2, -1]
+
+
+# ------------------------------------------------------------------ experts (App. E.2)
+
+def _swiglu_np(x, Wg, Wu, Wd):
+    g = x @ Wg.T
+    return ((g / (1.0 + np.exp(-g))) * (x @ Wu.T)) @ Wd.T
+
+
+def test_single_expert_top1_is_a_dense_swiglu_mlp():
+    """N = k = 1: the gate is Softmax of one logit = 1 and the layer is one dense gated MLP."""
+    cfg = synth.LayerConfig("t", T=20, d=24, N=1, k=1, m=40, dtype="fp32")
+    L = synth.make_layer(cfg, seed=3)
+    r = oracle.route_predict(L["x"], L["W_router"], L["W_pred"], 1)
+    assert np.all(r["gates"] == 1.0) and np.all(r["idx"] == 0)
+    out = oracle.moe_forward(L["x"], r["idx"], r["gates"], L["W_gate"], L["W_up"], L["W_down"])
+    ref = _swiglu_np(_f64(L["x"]), _f64(L["W_gate"][0]), _f64(L["W_up"][0]), _f64(L["W_down"][0]))
+    assert np.max(np.abs(out - ref)) <= 1e-12 * np.max(np.abs(ref))
+
+
+def test_permutation_matrix_experts_have_a_closed_form():
+    """Wg, Wu, Wd permutation matrices (m = d): y = P3 (silu(P1 x) * (P2 x)) exactly; the
+    permutations are not involutions, so any transposed weight read changes the result."""
+    d = 7
+    p1, p2, p3 = [1, 2, 3, 4, 5, 6, 0], [3, 0, 6, 1, 4, 2, 5], [2, 4, 6, 1, 3, 5, 0]
+    def pm(p):
+        M = torch.zeros(d, d)
+        for r_, c in enumerate(p):
+            M[r_, c] = 1.0
+        return M
+    x = _rand((3, d), 80)
+    Wg, Wu, Wd = pm(p1)[None], pm(p2)[None], pm(p3)[None]
+    idx = np.zeros((3, 1), np.int32)
+    gates = np.array([[1.0], [0.5], [2.0]])
+    out = oracle.moe_forward(x, idx, gates, Wg, Wu, Wd)
+    for t in range(3):
+        xt = [float(v) for v in x[t]]
+        a = [xt[p1[j]] / (1.0 + math.exp(-xt[p1[j]])) * xt[p2[j]] for j in range(d)]
+        y = [a[p3[c]] for c in range(d)]
+        assert np.allclose(out[t], gates[t, 0] * np.array(y), rtol=1e-15, atol=1e-16)
+
+
+def test_zero_up_projection_gives_zero_output():
+    cfg = synth.LayerConfig("t", T=10, d=16, N=4, k=2, m=8, dtype="fp32")
+    L = synth.make_layer(cfg, seed=4)
+    r = oracle.route_predict(L["x"], L["W_router"], L["W_pred"], 2)
+    out = oracle.moe_forward(L["x"], r["idx"], r["gates"], L["W_gate"],
+                             torch.zeros_like(L["W_up"]), L["W_down"])
+    assert np.all(out == 0.0)
+
+
+def test_dense_uniform_mixture_is_the_expert_mean():
+    """k = N with W = W_p = 0: every gate is 1/N and the layer is the mean of all experts."""
+    cfg = synth.LayerConfig("t", T=6, d=16, N=4, k=4, m=8, dtype="fp32")
+    L = synth.make_layer(cfg, seed=5)
+    Z = torch.zeros(4, 16)
+    r = oracle.route_predict(L["x"], Z, Z, 4)
+    out = oracle.moe_forward(L["x"], r["idx"], r["gates"], L["W_gate"], L["W_up"], L["W_down"])
+    x = _f64(L["x"])
+    ref = sum(_swiglu_np(x, _f64(L["W_gate"][e]), _f64(L["W_up"][e]), _f64(L["W_down"][e]))
+              for e in range(4)) / 4
+    assert np.max(np.abs(out - ref)) <= 1e-12 * np.max(np.abs(ref))
+
+
+def test_routed_sum_follows_slot_gates_and_experts():
+    """Two-slot routing against per-expert dense MLPs (catches a wrong expert offset or a gate
+    applied to the wrong slot)."""
+    cfg = synth.LayerConfig("t", T=9, d=16, N=5, k=2, m=12, dtype="fp32")
+    L = synth.make_layer(cfg, seed=6)
+    rng = np.random.default_rng(0)
+    idx = np.stack([rng.permutation(5)[:2] for _ in range(9)]).astype(np.int32)
+    gates = rng.random((9, 2))
+    out = oracle.moe_forward(L["x"], idx, gates, L["W_gate"], L["W_up"], L["W_down"])
+    x = _f64(L["x"])
+    for t in range(9):
+        ref = sum(gates[t, s] * _swiglu_np(x[t:t + 1], _f64(L["W_gate"][e]), _f64(L["W_up"][e]),
+                                            _f64(L["W_down"][e]))[0]
+                  for s, e in enumerate(idx[t]))
+        assert np.max(np.abs(out[t] - ref)) <= 1e-12 * np.max(np.abs(ref))
+
+
+def test_shared_expert_alone_when_routed_gates_are_zero():
+    cfg = synth.LayerConfig("t", T=8, d=16, N=4, k=2, m=8, n_shared=1, dtype="fp32")
+    L = synth.make_layer(cfg, seed=7)
+    r = oracle.route_predict(L["x"], L["W_router"], L["W_pred"], 2)
+    out = oracle.moe_forward(L["x"], r["idx"], np.zeros((8, 2)), L["W_gate"], L["W_up"],
+                             L["W_down"], L["Ws_gate"], L["Ws_up"], L["Ws_down"])
+    ref = _swiglu_np(_f64(L["x"]), _f64(L["Ws_gate"][0]), _f64(L["Ws_up"][0]),
+                     _f64(L["Ws_down"][0]))
+    assert np.max(np.abs(out - ref)) <= 1e-12 * np.max(np.abs(ref))
+
+
+def test_rollout_then_replay_of_its_route_reproduces_the_output():
+    """W_p = 0 and the same router: replaying the recorded route gives the rollout output."""
+    cfg = synth.LayerConfig("t", T=24, d=16, N=6, k=2, m=8, dtype="fp32")
+    L = synth.make_layer(cfg, seed=8)
+    Z = torch.zeros_like(L["W_pred"])
+    r = oracle.route_predict(L["x"], L["W_router"], Z, 2)
+    rep = oracle.route_replay(L["x"], L["W_router"], r["idx"])
+    o1 = oracle.moe_forward(L["x"], r["idx"], r["gates"], L["W_gate"], L["W_up"], L["W_down"])
+    o2 = oracle.moe_forward(L["x"], r["idx"], rep["gates"], L["W_gate"], L["W_up"], L["W_down"])
+    assert np.array_equal(o1, o2)
+
+
+def test_token_subset_matches_full_run_and_bf16_inputs_widen_exactly():
+    cfg = synth.LayerConfig("t", T=12, d=16, N=4, k=2, m=8, dtype="bf16")
+    L = synth.make_layer(cfg, seed=9)
+    r = oracle.route_predict(L["x"], L["W_router"], L["W_pred"], 2)
+    full = oracle.moe_forward(L["x"], r["idx"], r["gates"], L["W_gate"], L["W_up"], L["W_down"])
+    sub = oracle.moe_forward(L["x"], r["idx"], r["gates"], L["W_gate"], L["W_up"], L["W_down"],
+                             tokens=[11, 0, 5])
+    assert np.array_equal(sub, full[[11, 0, 5]])
+    # bf16 -> double widening is exact: same values given as fp32 give identical results
+    r32 = oracle.route_predict(L["x"].float(), L["W_router"].float(), L["W_pred"].float(), 2)
+    assert np.array_equal(r32["logits"], r["logits"]) and np.array_equal(r32["idx"], r["idx"])
