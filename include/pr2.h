@@ -1,0 +1,157 @@
+/*
+ * pr2.h - C ABI of the Pr^2 (Predictive Routing Replay) MoE-layer forward for GB300 (sm_103a).
+ *
+ * The layer has two modes (Sec. 4.1 of arxiv 2606.00395):
+ *   rollout:  pr2_route_predict  then  pr2_moe_forward   (Eqs. pr2_predict, pr2_route,
+ *             pr2_old_output; Algorithm 1 rollout steps, Algorithm 2)
+ *   training: pr2_route_replay   then  pr2_moe_forward   (Sec. 4.1 "Replay During Training",
+ *             Eq. pr2_output; Algorithm 1 replay steps, Algorithm 3)
+ *
+ * Conventions shared by every entry point:
+ *  - Every tensor argument is a DEVICE pointer to a contiguous row-major buffer owned by the
+ *    caller; the library allocates nothing, keeps no state between calls and is re-entrant per
+ *    stream.  All work is enqueued asynchronously on `stream` (a cudaStream_t; NULL = legacy
+ *    default stream).  Pointers must be 16-byte aligned.
+ *  - h, the weights and the layer output share dims->dtype (PR2_FP32 or PR2_BF16).  Gates,
+ *    logits and probabilities are always fp32; expert indices are int32 (App. E.2 stores the
+ *    replay indices as int32).
+ *  - Weights are stored [out, in]: W_router[e*d + i] is entry (i, e) of the paper's d x N
+ *    router matrix W, so the logits p = h W of Sec. 4.1 are p[t,e] = sum_i h[t,i] W_router[e*d+i].
+ *    W_pred has the same layout for the evolution predictor W_p.  Expert weights are stacked:
+ *    W_gate, W_up [N, m, d]; W_down [N, d, m]; shared experts Ws_* the same with n_shared rows.
+ *  - Host-detectable problems (NULL pointer, unsupported shape, short workspace) return an
+ *    error before anything is launched.  Data-dependent problems found on the device (a replay
+ *    index outside [0, N) or repeated within a token; a bounded device wait that ran out) are
+ *    OR-ed into the caller's device status word as PR2_STATUS_* bits; the offending slot then
+ *    contributes nothing.  With PR2_F_SYNC_STATUS in dims->flags the call synchronises the
+ *    stream, reads the status word and returns PR2_ERR_BAD_INDEX / PR2_ERR_TIMEOUT.  No C++
+ *    exception crosses this ABI and no kernel traps.
+ *  - Supported shapes: 1 <= k <= min(N, 32).  PR2_FP32 runs exact-fp32 SIMT kernels (N <= 256).
+ *    PR2_BF16 runs tcgen05 tensor-core kernels (fp32 accumulation) and needs d % 64 == 0,
+ *    m % 64 == 0, N % 16 == 0, N <= 256 and k <= 8.  Anything else returns PR2_ERR_UNSUPPORTED.
+ */
+#ifndef PR2_H
+#define PR2_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    PR2_OK = 0,
+    PR2_ERR_INVALID_ARG = 1,  /* NULL pointer, k > N, T < 0, ...                             */
+    PR2_ERR_UNSUPPORTED = 2,  /* valid but outside the shapes/dtypes listed above              */
+    PR2_ERR_CUDA = 3,         /* a CUDA runtime call or launch failed                          */
+    PR2_ERR_BAD_INDEX = 4,    /* (PR2_F_SYNC_STATUS only) invalid replay index seen on device  */
+    PR2_ERR_TIMEOUT = 5,      /* (PR2_F_SYNC_STATUS only) a bounded device wait ran out        */
+    PR2_ERR_WORKSPACE = 6     /* workspace NULL or smaller than pr2_moe_workspace_bytes()      */
+} pr2_status;
+
+typedef enum { PR2_FP32 = 0, PR2_BF16 = 1 } pr2_dtype;
+
+/* dims->flags bits */
+#define PR2_F_SYNC_STATUS 0x1u /* synchronise `stream` and turn the status word into a code */
+
+/* device status word bits (OR-ed in by the kernels; the caller zeroes the word) */
+#define PR2_STATUS_BAD_INDEX 0x1
+#define PR2_STATUS_TIMEOUT 0x2
+
+/* A token counts as a near tie when its k-th and (k+1)-th predicted probabilities differ by
+ * less than this (the top-k margin Delta_k of Lemma topk_regret, App. B). */
+#define PR2_NEAR_TIE_GAP 1e-4
+
+/* Problem size of one MoE layer: T tokens, d = d_model, N routed experts, top-k, m = expert
+ * hidden size (d_ff), n_shared always-on shared experts (App. E.2, "s"). */
+typedef struct {
+    int64_t T;
+    int32_t d, N, k, m, n_shared;
+    int32_t dtype;   /* pr2_dtype */
+    uint32_t flags;  /* PR2_F_* */
+} pr2_dims;
+
+/*
+ * Rollout routing, Eqs. pr2_predict and pr2_route (Sec. 4.1 "Route Prediction During Rollout"),
+ * with the route record of Algorithm 2:
+ *     p_old = h W_old,  b = h W_p,  rho_hat = Softmax(p_old + b),  I_hat = TopK(rho_hat, k).
+ *  h          [T, d]  dtype     router input h_old
+ *  W_router   [N, d]  dtype     old-snapshot router (transposed W_old)
+ *  W_pred     [N, d]  dtype     evolution predictor (transposed W_p)
+ *  idx        [T, k]  int32     out: I_hat, slots by descending rho_hat, ties to the lower index
+ *  gates      [T, k]  fp32      out: rho_hat at idx (full-softmax probability, not renormalised)
+ *  logits_old [T, N]  fp32      out, nullable: p_old, the feature-cache logits of Algorithm 2
+ *  near_tie   [1]     int64     in/out, nullable: += #tokens whose rho_hat_(k) - rho_hat_(k+1)
+ *                               < PR2_NEAR_TIE_GAP (k < N)
+ *  status_dev [1]     int32     in/out, nullable: PR2_STATUS_* bits
+ */
+pr2_status pr2_route_predict(const pr2_dims* dims, const void* h, const void* W_router,
+                             const void* W_pred, int32_t* idx, float* gates, float* logits_old,
+                             int64_t* near_tie, int32_t* status_dev, void* stream);
+
+/*
+ * Training-time replay gates, Sec. 4.1 "Replay During Training" (Algorithm 3, first step):
+ *     rho = Softmax(h W),  gates[t,s] = rho[t, idx[t,s]];  no fresh top-k, no predictor.
+ *  h [T,d], W_router [N,d] (current router, dtype); idx [T,k] int32 the cached route;
+ *  gates [T,k] fp32 out (0 for an invalid slot); probs [T,N] fp32 out, nullable: the full rho;
+ *  status_dev nullable (PR2_STATUS_BAD_INDEX for an index outside [0,N) or repeated in a token).
+ */
+pr2_status pr2_route_replay(const pr2_dims* dims, const void* h, const void* W_router,
+                            const int32_t* idx, float* gates, float* probs, int32_t* status_dev,
+                            void* stream);
+
+/* Optional stage markers of pr2_moe_forward for profiling: each non-NULL member is a
+ * cudaEvent_t (created by the caller on the current device) that the call records on `stream`
+ * at that point of the launch sequence.  NULL members and a NULL struct pointer are ignored. */
+typedef struct {
+    void* start;         /* before dispatch                                              */
+    void* dispatched;    /* after histogram, scan, stable placement and row gather       */
+    void* gate_up_done;  /* after the gate/up + SwiGLU GEMM(s) (routed, then shared)     */
+    void* down_done;     /* after the down GEMM(s)                                       */
+    void* end;           /* after the gate-weighted combine                              */
+} pr2_stage_events;
+
+/* Bytes of device workspace pr2_moe_forward needs for `dims` (0 for invalid dims). */
+size_t pr2_moe_workspace_bytes(const pr2_dims* dims);
+
+/*
+ * MoE layer output on a given route, Eq. pr2_old_output (rollout gates rho_hat[idx]) and
+ * Eq. pr2_output (replay gates rho[idx]); experts are gated MLPs (App. E.2) with SwiGLU:
+ *     out[t] = sum_{s<k} gates[t,s] * E_{idx[t,s]}(h_t) + sum_{j<n_shared} E^shared_j(h_t),
+ *     E(x) = W_down (silu(W_gate x) * (W_up x)).
+ *  h [T,d] dtype; idx [T,k] int32; gates [T,k] fp32; W_gate, W_up [N,m,d]; W_down [N,d,m];
+ *  Ws_gate, Ws_up [n_shared,m,d], Ws_down [n_shared,d,m] (NULL iff n_shared == 0);
+ *  out [T,d] dtype (written, fp32 accumulation, rounded once);
+ *  counts [N] int32 out, nullable: tokens per expert (valid slots only);
+ *  perm [T*k] int32 out, nullable: flat slot ids t*k+s grouped by expert, stable in slot order
+ *      (entries past sum(counts) are unspecified);
+ *  workspace/ws_bytes: device scratch of at least pr2_moe_workspace_bytes(dims) bytes, 256-byte
+ *      aligned, owned by the caller and reused freely between calls on the same stream;
+ *  status_dev nullable (a status word inside the workspace is used when NULL);
+ *  events nullable: stage markers recorded for profiling (see pr2_stage_events).
+ */
+pr2_status pr2_moe_forward(const pr2_dims* dims, const void* h, const int32_t* idx,
+                           const float* gates, const void* W_gate, const void* W_up,
+                           const void* W_down, const void* Ws_gate, const void* Ws_up,
+                           const void* Ws_down, void* out, int32_t* counts, int32_t* perm,
+                           void* workspace, size_t ws_bytes, int32_t* status_dev,
+                           const pr2_stage_events* events, void* stream);
+
+/* Static, human-readable name of a status code. */
+const char* pr2_strerror(pr2_status s);
+
+/*
+ * Self-test of the bounded device wait used by every pipelined kernel (no paper counterpart):
+ * launches one CTA that waits on a barrier nothing will ever complete, gives up after
+ * `timeout_ns` nanoseconds, ORs PR2_STATUS_TIMEOUT into status_dev[0] and returns normally.
+ * timeout_ns must lie in [1e3, 1e9].  Lets a caller check that a stalled pipeline reports an
+ * error instead of hanging.
+ */
+pr2_status pr2_selftest_wait_timeout(int32_t* status_dev, int64_t timeout_ns, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PR2_H */

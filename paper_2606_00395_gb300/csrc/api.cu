@@ -1,0 +1,351 @@
+// C ABI of the Pr^2 MoE layer (declared in include/pr2.h): argument validation, workspace
+// layout, TMA descriptor encoding and the launch sequence of each entry point.
+#include <cudaTypedefs.h>
+
+#include <cstring>
+
+#include "pr2_device.cuh"
+#include "pr2_internal.h"
+
+namespace pr2 {
+namespace {
+
+// ---- TMA descriptor encoding through the driver entry point (no libcuda link needed) ------
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (fn == nullptr) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor [outer, inner] (row-major, row pitch = inner elements), 128-byte swizzled
+// boxes of box_inner x box_outer elements.
+bool make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
+                    uint32_t box_inner, uint32_t box_outer) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+int num_sms_of_current_device() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return n;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+pr2_status check_dims(const pr2_dims* dm) {
+  if (dm == nullptr) return PR2_ERR_INVALID_ARG;
+  if (dm->T < 0 || dm->d <= 0 || dm->N <= 0 || dm->k <= 0 || dm->k > dm->N || dm->m <= 0 ||
+      dm->n_shared < 0)
+    return PR2_ERR_INVALID_ARG;
+  if (dm->dtype != PR2_FP32 && dm->dtype != PR2_BF16) return PR2_ERR_INVALID_ARG;
+  if (dm->T * static_cast<int64_t>(dm->k) > (int64_t{1} << 30)) return PR2_ERR_UNSUPPORTED;
+  if (dm->N > kMaxExperts) return PR2_ERR_UNSUPPORTED;
+  if (dm->dtype == PR2_FP32) {
+    if (dm->k > kMaxTopKSimt || dm->d % 4 != 0) return PR2_ERR_UNSUPPORTED;
+  } else {
+    if (dm->k > kMaxTopK || dm->d % 64 != 0 || dm->m % 64 != 0 || dm->N % 16 != 0)
+      return PR2_ERR_UNSUPPORTED;
+  }
+  return PR2_OK;
+}
+
+size_t esize(const pr2_dims& dm) { return dm.dtype == PR2_FP32 ? 4 : 2; }
+
+// ---- workspace layout of pr2_moe_forward ----------------------------------------------------
+struct Workspace {
+  int32_t* status;
+  int32_t* blk_hist;
+  int32_t* counts;
+  int32_t* offsets;
+  int32_t* perm;
+  int32_t* inv;
+  int32_t* num_tiles;
+  TileEntry* tiles;
+  TileEntry* stiles1;
+  TileEntry* stiles2;
+  void* xperm;
+  void* hbuf;
+  void* ybuf;
+  void* hs;
+  void* ys;
+  int nblk, max_tiles, shared_tiles;
+  size_t total;
+};
+
+Workspace carve(const pr2_dims& dm, uint8_t* base) {
+  Workspace w{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) -> uint8_t* {
+    uint8_t* p = base ? base + off : nullptr;
+    off += (bytes + 255) & ~size_t{255};
+    return p;
+  };
+  const int64_t F = dm.T * dm.k;
+  const size_t es = esize(dm);
+  w.nblk = static_cast<int>((F + kDispatchChunk - 1) / kDispatchChunk);
+  w.max_tiles = static_cast<int>(F / kTileM + dm.N + 1);
+  const int mt_T = static_cast<int>((dm.T + kTileM - 1) / kTileM);
+  w.shared_tiles = dm.n_shared * mt_T;
+  w.status = reinterpret_cast<int32_t*>(take(sizeof(int32_t)));
+  w.blk_hist = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (size_t)w.nblk * dm.N));
+  w.counts = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * dm.N));
+  w.offsets = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (dm.N + 1)));
+  w.perm = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * F));
+  w.inv = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * F));
+  w.num_tiles = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * 2));
+  w.tiles = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * w.max_tiles));
+  w.stiles1 = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * (w.shared_tiles + 1)));
+  w.stiles2 = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * (w.shared_tiles + 1)));
+  w.xperm = take(es * F * dm.d);
+  w.hbuf = take(es * F * dm.m);
+  w.ybuf = take(es * F * dm.d);
+  w.hs = take(es * dm.n_shared * dm.T * dm.m);
+  w.ys = take(es * dm.n_shared * dm.T * dm.d);
+  w.total = off;
+  return w;
+}
+
+pr2_status finish(cudaError_t err, uint32_t flags, int32_t* status_dev, cudaStream_t st) {
+  if (err != cudaSuccess) return PR2_ERR_CUDA;
+  if (flags & PR2_F_SYNC_STATUS) {
+    if (status_dev == nullptr) return PR2_ERR_INVALID_ARG;
+    int32_t hst = 0;
+    if (cudaMemcpyAsync(&hst, status_dev, sizeof(hst), cudaMemcpyDeviceToHost, st) != cudaSuccess)
+      return PR2_ERR_CUDA;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return PR2_ERR_CUDA;
+    if (hst & PR2_STATUS_TIMEOUT) return PR2_ERR_TIMEOUT;
+    if (hst & PR2_STATUS_BAD_INDEX) return PR2_ERR_BAD_INDEX;
+  }
+  return PR2_OK;
+}
+
+pr2_status route_common(const pr2_dims* dims, bool predict, const void* h, const void* W,
+                        const void* Wp, const int32_t* idx_in, int32_t* idx_out, float* gates,
+                        float* aux, int64_t* near_tie, int32_t* status_dev, void* stream) {
+  pr2_status s = check_dims(dims);
+  if (s != PR2_OK) return s;
+  const pr2_dims& dm = *dims;
+  if (dm.T == 0) return PR2_OK;  // nothing to route; empty tensors may have NULL data
+  if (h == nullptr || W == nullptr || gates == nullptr) return PR2_ERR_INVALID_ARG;
+  if (predict && (Wp == nullptr || idx_out == nullptr)) return PR2_ERR_INVALID_ARG;
+  if (!predict && idx_in == nullptr) return PR2_ERR_INVALID_ARG;
+  if ((dm.flags & PR2_F_SYNC_STATUS) && status_dev == nullptr) return PR2_ERR_INVALID_ARG;
+  if (!aligned16(h) || !aligned16(W) || (Wp && !aligned16(Wp)) || (aux && !aligned16(aux)))
+    return PR2_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t err;
+  if (dm.dtype == PR2_FP32) {
+    err = launch_route_simt(dm, predict, static_cast<const float*>(h),
+                            static_cast<const float*>(W), static_cast<const float*>(Wp), idx_in,
+                            idx_out, gates, aux, near_tie, status_dev, st);
+  } else {
+    if (dm.T > (int64_t{1} << 30)) return PR2_ERR_UNSUPPORTED;
+    CUtensorMap tm_h, tm_w, tm_wp;
+    if (!make_tmap_bf16(&tm_h, h, dm.d, dm.T, 64, kTileM) ||
+        !make_tmap_bf16(&tm_w, W, dm.d, dm.N, 64, dm.N))
+      return PR2_ERR_CUDA;
+    if (predict) {
+      if (!make_tmap_bf16(&tm_wp, Wp, dm.d, dm.N, 64, dm.N)) return PR2_ERR_CUDA;
+    } else {
+      tm_wp = tm_w;
+    }
+    RouteTcArgs a{static_cast<int>(dm.T), dm.d, dm.N, dm.k, idx_in, idx_out,
+                  gates, aux, near_tie, status_dev};
+    err = launch_route_tc(predict, tm_h, tm_w, tm_wp, a, st);
+  }
+  return finish(err, dm.flags, status_dev, st);
+}
+
+}  // namespace
+}  // namespace pr2
+
+using namespace pr2;
+
+extern "C" {
+
+pr2_status pr2_route_predict(const pr2_dims* dims, const void* h, const void* W_router,
+                             const void* W_pred, int32_t* idx, float* gates, float* logits_old,
+                             int64_t* near_tie, int32_t* status_dev, void* stream) {
+  return route_common(dims, true, h, W_router, W_pred, nullptr, idx, gates, logits_old, near_tie,
+                      status_dev, stream);
+}
+
+pr2_status pr2_route_replay(const pr2_dims* dims, const void* h, const void* W_router,
+                            const int32_t* idx, float* gates, float* probs, int32_t* status_dev,
+                            void* stream) {
+  return route_common(dims, false, h, W_router, nullptr, idx, nullptr, gates, probs, nullptr,
+                      status_dev, stream);
+}
+
+size_t pr2_moe_workspace_bytes(const pr2_dims* dims) {
+  if (check_dims(dims) != PR2_OK) return 0;
+  return carve(*dims, nullptr).total;
+}
+
+pr2_status pr2_moe_forward(const pr2_dims* dims, const void* h, const int32_t* idx,
+                           const float* gates, const void* W_gate, const void* W_up,
+                           const void* W_down, const void* Ws_gate, const void* Ws_up,
+                           const void* Ws_down, void* out, int32_t* counts, int32_t* perm,
+                           void* workspace, size_t ws_bytes, int32_t* status_dev,
+                           const pr2_stage_events* events, void* stream) {
+  pr2_status s = check_dims(dims);
+  if (s != PR2_OK) return s;
+  const pr2_dims& dm = *dims;
+  if (dm.T == 0) return PR2_OK;  // empty layer: nothing to write
+  if (h == nullptr || idx == nullptr || gates == nullptr || W_gate == nullptr ||
+      W_up == nullptr || W_down == nullptr || out == nullptr)
+    return PR2_ERR_INVALID_ARG;
+  if (dm.n_shared > 0 && (Ws_gate == nullptr || Ws_up == nullptr || Ws_down == nullptr))
+    return PR2_ERR_INVALID_ARG;
+  if (dm.n_shared == 0 && (Ws_gate != nullptr || Ws_up != nullptr || Ws_down != nullptr))
+    return PR2_ERR_INVALID_ARG;
+  const void* ptrs[] = {h, W_gate, W_up, W_down, out};
+  for (const void* p : ptrs)
+    if (!aligned16(p)) return PR2_ERR_INVALID_ARG;
+  if (dm.n_shared > 0 && (!aligned16(Ws_gate) || !aligned16(Ws_up) || !aligned16(Ws_down)))
+    return PR2_ERR_INVALID_ARG;
+  const Workspace probe = carve(dm, nullptr);
+  if (workspace == nullptr || ws_bytes < probe.total ||
+      (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+    return PR2_ERR_WORKSPACE;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const Workspace w = carve(dm, static_cast<uint8_t*>(workspace));
+  int32_t* status = status_dev ? status_dev : w.status;
+  const int num_sms = num_sms_of_current_device();
+  if (num_sms <= 0) return PR2_ERR_CUDA;
+  cudaError_t err = cudaSuccess;
+  if (status_dev == nullptr) err = cudaMemsetAsync(w.status, 0, sizeof(int32_t), st);
+  if (err != cudaSuccess) return PR2_ERR_CUDA;
+  auto mark = [&](void* ev) {
+    if (ev != nullptr && err == cudaSuccess)
+      err = cudaEventRecord(static_cast<cudaEvent_t>(ev), st);
+  };
+  mark(events ? events->start : nullptr);
+
+  const int es = static_cast<int>(esize(dm));
+  DispatchArgs da{idx,       dm.T,       dm.k,      dm.N,    dm.d,   es,     dm.n_shared,
+                  w.blk_hist, w.counts,  w.offsets, w.perm,  w.inv,  w.tiles, w.num_tiles,
+                  w.stiles1, w.stiles2,  h,         w.xperm, status};
+  if (err == cudaSuccess) err = launch_dispatch(da, num_sms, st);
+  mark(events ? events->dispatched : nullptr);
+  if (err != cudaSuccess) return PR2_ERR_CUDA;
+
+  const int64_t F = dm.T * dm.k;
+  GemmArgs g1{w.tiles, w.num_tiles, w.max_tiles, dm.d, dm.m, dm.m, w.hbuf, status};
+  GemmArgs g2{w.tiles, w.num_tiles, w.max_tiles, dm.m, dm.d, dm.d, w.ybuf, status};
+  GemmArgs s1{w.stiles1, w.num_tiles + 1, w.shared_tiles, dm.d, dm.m, dm.m, w.hs, status};
+  GemmArgs s2{w.stiles2, w.num_tiles + 1, w.shared_tiles, dm.m, dm.d, dm.d, w.ys, status};
+  if (dm.dtype == PR2_BF16) {
+    CUtensorMap a1, b1g, b1u, a2, b2, sa1, sb1g, sb1u, sa2, sb2;
+    bool ok = make_tmap_bf16(&a1, w.xperm, dm.d, F, 64, kTileM) &&
+              make_tmap_bf16(&b1g, W_gate, dm.d, (uint64_t)dm.N * dm.m, 64, 128) &&
+              make_tmap_bf16(&b1u, W_up, dm.d, (uint64_t)dm.N * dm.m, 64, 128) &&
+              make_tmap_bf16(&a2, w.hbuf, dm.m, F, 64, kTileM) &&
+              make_tmap_bf16(&b2, W_down, dm.m, (uint64_t)dm.N * dm.d, 64, 256);
+    if (ok && dm.n_shared > 0) {
+      ok = make_tmap_bf16(&sa1, h, dm.d, dm.T, 64, kTileM) &&
+           make_tmap_bf16(&sb1g, Ws_gate, dm.d, (uint64_t)dm.n_shared * dm.m, 64, 128) &&
+           make_tmap_bf16(&sb1u, Ws_up, dm.d, (uint64_t)dm.n_shared * dm.m, 64, 128) &&
+           make_tmap_bf16(&sa2, w.hs, dm.m, (uint64_t)dm.n_shared * dm.T, 64, kTileM) &&
+           make_tmap_bf16(&sb2, Ws_down, dm.m, (uint64_t)dm.n_shared * dm.d, 64, 256);
+    }
+    if (!ok) return PR2_ERR_CUDA;
+    err = launch_expert_tc(true, a1, b1g, b1u, g1, num_sms, st);
+    if (err == cudaSuccess && dm.n_shared > 0)
+      err = launch_expert_tc(true, sa1, sb1g, sb1u, s1, num_sms, st);
+    mark(events ? events->gate_up_done : nullptr);
+    if (err == cudaSuccess) err = launch_expert_tc(false, a2, b2, b2, g2, num_sms, st);
+    if (err == cudaSuccess && dm.n_shared > 0)
+      err = launch_expert_tc(false, sa2, sb2, sb2, s2, num_sms, st);
+    mark(events ? events->down_done : nullptr);
+  } else {
+    err = launch_expert_simt(true, static_cast<const float*>(w.xperm),
+                             static_cast<const float*>(W_gate), static_cast<const float*>(W_up),
+                             g1, st);
+    if (err == cudaSuccess && dm.n_shared > 0)
+      err = launch_expert_simt(true, static_cast<const float*>(h),
+                               static_cast<const float*>(Ws_gate),
+                               static_cast<const float*>(Ws_up), s1, st);
+    mark(events ? events->gate_up_done : nullptr);
+    if (err == cudaSuccess)
+      err = launch_expert_simt(false, static_cast<const float*>(w.hbuf),
+                               static_cast<const float*>(W_down), nullptr, g2, st);
+    if (err == cudaSuccess && dm.n_shared > 0)
+      err = launch_expert_simt(false, static_cast<const float*>(w.hs),
+                               static_cast<const float*>(Ws_down), nullptr, s2, st);
+    mark(events ? events->down_done : nullptr);
+  }
+  if (err != cudaSuccess) return PR2_ERR_CUDA;
+
+  CombineArgs ca{w.ybuf, dm.n_shared > 0 ? w.ys : nullptr, w.inv, gates, dm.T, dm.k, dm.d,
+                 dm.n_shared, dm.dtype == PR2_BF16 ? 1 : 0, out};
+  err = launch_combine(ca, num_sms, st);
+  mark(events ? events->end : nullptr);
+  if (err == cudaSuccess && counts != nullptr)
+    err = cudaMemcpyAsync(counts, w.counts, sizeof(int32_t) * dm.N, cudaMemcpyDeviceToDevice, st);
+  if (err == cudaSuccess && perm != nullptr)
+    err = cudaMemcpyAsync(perm, w.perm, sizeof(int32_t) * F, cudaMemcpyDeviceToDevice, st);
+  return finish(err, dm.flags, status, st);
+}
+
+const char* pr2_strerror(pr2_status s) {
+  switch (s) {
+    case PR2_OK: return "ok";
+    case PR2_ERR_INVALID_ARG: return "invalid argument";
+    case PR2_ERR_UNSUPPORTED: return "unsupported shape or dtype";
+    case PR2_ERR_CUDA: return "CUDA error";
+    case PR2_ERR_BAD_INDEX: return "invalid expert index in route";
+    case PR2_ERR_TIMEOUT: return "device wait timed out";
+    case PR2_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+  }
+  return "unknown status";
+}
+
+pr2_status pr2_selftest_wait_timeout(int32_t* status_dev, int64_t timeout_ns, void* stream) {
+  if (status_dev == nullptr || timeout_ns < 1000 || timeout_ns > 1000000000) return PR2_ERR_INVALID_ARG;
+  cudaError_t err = launch_wait_selftest(status_dev, timeout_ns, static_cast<cudaStream_t>(stream));
+  return err == cudaSuccess ? PR2_OK : PR2_ERR_CUDA;
+}
+
+}  // extern "C"
+
+namespace pr2 {
+namespace {
+// One thread waits on an mbarrier that expects an arrival nobody makes; the bounded wait gives
+// up after timeout_ns and records PR2_STATUS_TIMEOUT.
+__global__ void wait_selftest_kernel(int32_t* status, int64_t timeout_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0)
+    mbar_wait_slow(&bar, 0, &abort_flag, status, static_cast<uint64_t>(timeout_ns));
+}
+}  // namespace
+
+cudaError_t launch_wait_selftest(int32_t* status, int64_t timeout_ns, cudaStream_t st) {
+  wait_selftest_kernel<<<1, 32, 0, st>>>(status, timeout_ns);
+  return cudaGetLastError();
+}
+}  // namespace pr2

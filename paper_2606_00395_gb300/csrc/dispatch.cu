@@ -1,0 +1,262 @@
+// Dispatch of (token, slot) pairs to experts and the gate-weighted combine.
+//
+// Dispatch ("dispatch to experts", Algorithm 1) is a stable counting sort of the flat slot ids
+// f = t*k + s by expert id, deterministic and bit-exact:
+//   1. hist   - one block per 256 slots: validate each slot (expert in [0,N), not repeated in
+//               its token) and count per expert in shared memory -> blk_hist[b][e].
+//   2. scan   - one block: per expert an exclusive scan over blocks (in place), the expert
+//               totals (counts), their exclusive scan (offsets), the M-tile table of the
+//               grouped GEMM, and the static tile tables of the shared experts.
+//   3. place  - one block per 256 slots again: per-warp counts via __match_any_sync, a scan
+//               over the 8 warps, then rank = popc(lanes below with the same expert):
+//               perm[offsets[e] + r] = f, inv[f] = its position (-1 for an invalid slot).
+//   4. gather - X[p, :] = h[perm[p] / k, :], 16-byte vectors, one warp per row.
+// Combine (the sums of Eqs. pr2_old_output / pr2_output):
+//   out[t, :] = sum_s gates[t,s] * Y[inv[t*k+s], :] + sum_j Ys[j, t, :], fp32 accumulation.
+#include "pr2_device.cuh"
+#include "pr2_internal.h"
+
+namespace pr2 {
+namespace {
+
+constexpr int kWarps = kDispatchChunk / 32;
+
+__device__ __forceinline__ bool slot_valid(const int32_t* __restrict__ idx, int64_t f, int k, int N,
+                                           int* e_out) {
+  const int e = idx[f];
+  bool ok = e >= 0 && e < N;
+  const int64_t base = f - (f % k);
+  for (int64_t f2 = base; ok && f2 < f; ++f2)
+    if (idx[f2] == e) ok = false;
+  *e_out = ok ? e : -1;
+  return ok;
+}
+
+__global__ void __launch_bounds__(kDispatchChunk)
+    hist_kernel(const int32_t* __restrict__ idx, int64_t F, int k, int N,
+                int32_t* __restrict__ blk_hist, int32_t* status) {
+  __shared__ int hist[kMaxExpertsDispatch];
+  for (int e = threadIdx.x; e < N; e += blockDim.x) hist[e] = 0;
+  __syncthreads();
+  const int64_t f = static_cast<int64_t>(blockIdx.x) * kDispatchChunk + threadIdx.x;
+  if (f < F) {
+    int e;
+    if (slot_valid(idx, f, k, N, &e))
+      atomicAdd(&hist[e], 1);
+    else if (status != nullptr)
+      atomicOr(status, PR2_STATUS_BAD_INDEX);
+  }
+  __syncthreads();
+  int32_t* out = blk_hist + static_cast<int64_t>(blockIdx.x) * N;
+  for (int e = threadIdx.x; e < N; e += blockDim.x) out[e] = hist[e];
+}
+
+// Exclusive block-wide scan of one int per thread (blockDim.x == 1024).
+__device__ __forceinline__ int block_exclusive_scan(int v, int* sh, int* total) {
+  const int tid = threadIdx.x;
+  sh[tid] = v;
+  __syncthreads();
+  for (int o = 1; o < 1024; o <<= 1) {
+    const int add = tid >= o ? sh[tid - o] : 0;
+    __syncthreads();
+    sh[tid] += add;
+    __syncthreads();
+  }
+  const int incl = sh[tid];
+  *total = sh[1023];
+  __syncthreads();
+  return incl - v;
+}
+
+__global__ void __launch_bounds__(1024)
+    scan_kernel(int32_t* __restrict__ blk_hist, int nblk, int N, int64_t T, int n_shared,
+                int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
+                TileEntry* __restrict__ tiles, int32_t* __restrict__ num_tiles,
+                TileEntry* __restrict__ stiles1, TileEntry* __restrict__ stiles2) {
+  __shared__ int sh[1024];
+  const int e = threadIdx.x;
+  int total = 0;
+  if (e < N) {
+    for (int b = 0; b < nblk; ++b) {
+      int32_t* p = blk_hist + static_cast<int64_t>(b) * N + e;
+      const int v = *p;
+      *p = total;
+      total += v;
+    }
+    counts[e] = total;
+  }
+  int all_rows, all_tiles;
+  const int off = block_exclusive_scan(e < N ? total : 0, sh, &all_rows);
+  const int ntile_e = e < N ? (total + kTileM - 1) / kTileM : 0;
+  const int tstart = block_exclusive_scan(ntile_e, sh, &all_tiles);
+  if (e < N) {
+    offsets[e] = off;
+    for (int b = 0; b < nblk; ++b) blk_hist[static_cast<int64_t>(b) * N + e] += off;
+    for (int j = 0; j < ntile_e; ++j) {
+      const int r0 = off + j * kTileM;
+      const int rows = (total - j * kTileM) < kTileM ? (total - j * kTileM) : kTileM;
+      tiles[tstart + j] = TileEntry{e, r0, rows, r0};
+    }
+  }
+  if (e == 0) {
+    offsets[N] = all_rows;
+    num_tiles[0] = all_tiles;
+  }
+  // Shared experts: every token, fixed tiles.  Gate/up reads h rows, down reads Hs rows.
+  const int mt_T = static_cast<int>((T + kTileM - 1) / kTileM);
+  for (int i = e; i < n_shared * mt_T; i += blockDim.x) {
+    const int j = i / mt_T, m = i - j * mt_T;
+    const int r0 = m * kTileM;
+    const int rows = (T - r0) < kTileM ? static_cast<int>(T - r0) : kTileM;
+    const int o0 = static_cast<int>(j * T) + r0;
+    stiles1[i] = TileEntry{j, r0, rows, o0};
+    stiles2[i] = TileEntry{j, o0, rows, o0};
+  }
+  if (e == 0) num_tiles[1] = n_shared * mt_T;
+}
+
+__global__ void __launch_bounds__(kDispatchChunk)
+    place_kernel(const int32_t* __restrict__ idx, int64_t F, int k, int N,
+                 const int32_t* __restrict__ blk_base, int32_t* __restrict__ perm,
+                 int32_t* __restrict__ inv) {
+  __shared__ int wcnt[kWarps][kMaxExpertsDispatch];
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int i = threadIdx.x; i < kWarps * N; i += blockDim.x) wcnt[i / N][i % N] = 0;
+  __syncthreads();
+  const int64_t f = static_cast<int64_t>(blockIdx.x) * kDispatchChunk + threadIdx.x;
+  int e = -1;
+  if (f < F) slot_valid(idx, f, k, N, &e);
+  const unsigned same = __match_any_sync(0xffffffffu, e);
+  if (e >= 0 && lane == __ffs(same) - 1) wcnt[w][e] = __popc(same);
+  __syncthreads();
+  const int32_t* base = blk_base + static_cast<int64_t>(blockIdx.x) * N;
+  for (int x = threadIdx.x; x < N; x += blockDim.x) {
+    int run = base[x];
+    for (int ww = 0; ww < kWarps; ++ww) {
+      const int c = wcnt[ww][x];
+      wcnt[ww][x] = run;
+      run += c;
+    }
+  }
+  __syncthreads();
+  if (f < F) {
+    if (e >= 0) {
+      const int pos = wcnt[w][e] + __popc(same & lanemask_lt());
+      perm[pos] = static_cast<int32_t>(f);
+      inv[f] = pos;
+    } else {
+      inv[f] = -1;
+    }
+  }
+}
+
+// X[p, :] = h[perm[p] / k, :] for p < offsets[N]; row_vec = 16-byte vectors per row.
+__global__ void __launch_bounds__(256)
+    gather_kernel(const uint4* __restrict__ h, const int32_t* __restrict__ perm,
+                  const int32_t* __restrict__ nrows_ptr, int k, int row_vec,
+                  uint4* __restrict__ X) {
+  const int nrows = *nrows_ptr;
+  const int lane = threadIdx.x & 31;
+  const int warp0 = static_cast<int>((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  const int nwarps = static_cast<int>((gridDim.x * blockDim.x) >> 5);
+  for (int p = warp0; p < nrows; p += nwarps) {
+    const int t = perm[p] / k;
+    const uint4* src = h + static_cast<int64_t>(t) * row_vec;
+    uint4* dst = X + static_cast<int64_t>(p) * row_vec;
+#pragma unroll 4
+    for (int v = lane; v < row_vec; v += 32) dst[v] = __ldg(src + v);
+  }
+}
+
+template <typename T, int V>  // V elements per 16-byte vector
+__global__ void __launch_bounds__(256)
+    combine_kernel(const T* __restrict__ Y, const T* __restrict__ Ys,
+                   const int32_t* __restrict__ inv, const float* __restrict__ gates, int64_t Tn,
+                   int k, int d, int n_shared, T* __restrict__ out) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp0 = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  const int nvec = d / V;
+  for (int64_t t = warp0; t < Tn; t += nwarps) {
+    int my_pos = -1;
+    float my_g = 0.f;
+    if (lane < k) {
+      my_pos = inv[t * k + lane];
+      my_g = gates[t * k + lane];
+    }
+    // The loop bound is warp-uniform so the shuffles below always see all 32 lanes.
+    for (int c0 = 0; c0 < nvec; c0 += 32) {
+      const int c = c0 + lane;
+      const bool act = c < nvec;
+      float acc[V];
+#pragma unroll
+      for (int j = 0; j < V; ++j) acc[j] = 0.f;
+      for (int s = 0; s < k; ++s) {
+        const int p = __shfl_sync(0xffffffffu, my_pos, s);
+        const float gs = __shfl_sync(0xffffffffu, my_g, s);
+        if (p < 0 || !act) continue;
+        const uint4 raw = __ldg(reinterpret_cast<const uint4*>(Y + static_cast<int64_t>(p) * d) + c);
+        const T* v = reinterpret_cast<const T*>(&raw);
+#pragma unroll
+        for (int j = 0; j < V; ++j) acc[j] = fmaf(gs, to_f32<T>(v[j]), acc[j]);
+      }
+      if (!act) continue;
+      for (int j2 = 0; j2 < n_shared; ++j2) {
+        const uint4 raw = __ldg(
+            reinterpret_cast<const uint4*>(Ys + (static_cast<int64_t>(j2) * Tn + t) * d) + c);
+        const T* v = reinterpret_cast<const T*>(&raw);
+#pragma unroll
+        for (int j = 0; j < V; ++j) acc[j] += to_f32<T>(v[j]);
+      }
+      uint4 o;
+      T* ov = reinterpret_cast<T*>(&o);
+#pragma unroll
+      for (int j = 0; j < V; ++j) ov[j] = from_f32<T>(acc[j]);
+      reinterpret_cast<uint4*>(out + t * d)[c] = o;
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st) {
+  const int64_t F = a.T * a.k;
+  const int nblk = static_cast<int>((F + kDispatchChunk - 1) / kDispatchChunk);
+  if (nblk > 0) {
+    hist_kernel<<<nblk, kDispatchChunk, 0, st>>>(a.idx, F, a.k, a.N, a.blk_hist, a.status);
+  }
+  scan_kernel<<<1, 1024, 0, st>>>(a.blk_hist, nblk, a.N, a.T, a.n_shared, a.counts, a.offsets,
+                                  a.tiles, a.num_tiles, a.stiles1, a.stiles2);
+  if (nblk > 0) {
+    place_kernel<<<nblk, kDispatchChunk, 0, st>>>(a.idx, F, a.k, a.N, a.blk_hist, a.perm,
+                                                  a.inv);
+    const int row_vec = a.d * a.esz / 16;
+    int64_t warps_needed = F;
+    int64_t blocks = (warps_needed + 7) / 8;
+    const int64_t cap = static_cast<int64_t>(num_sms) * 8;
+    if (blocks > cap) blocks = cap;
+    gather_kernel<<<static_cast<int>(blocks), 256, 0, st>>>(
+        static_cast<const uint4*>(a.h), a.perm, a.offsets + a.N, a.k, row_vec,
+        static_cast<uint4*>(a.xperm));
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st) {
+  if (a.T == 0) return cudaSuccess;
+  int64_t blocks = (a.T + 7) / 8;
+  const int64_t cap = static_cast<int64_t>(num_sms) * 8;
+  if (blocks > cap) blocks = cap;
+  if (a.bf16) {
+    combine_kernel<__nv_bfloat16, 8><<<static_cast<int>(blocks), 256, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(a.Y), static_cast<const __nv_bfloat16*>(a.Ys), a.inv,
+        a.gates, a.T, a.k, a.d, a.n_shared, static_cast<__nv_bfloat16*>(a.out));
+  } else {
+    combine_kernel<float, 4><<<static_cast<int>(blocks), 256, 0, st>>>(
+        static_cast<const float*>(a.Y), static_cast<const float*>(a.Ys), a.inv, a.gates, a.T,
+        a.k, a.d, a.n_shared, static_cast<float*>(a.out));
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace pr2

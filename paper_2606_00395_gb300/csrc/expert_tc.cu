@@ -1,0 +1,254 @@
+// Grouped expert GEMMs on the tcgen05 tensor cores (bf16 operands, fp32 accumulation in TMEM).
+//
+// The gated-MLP expert of App. E.2 with the SwiGLU activation, over the rows that dispatch
+// grouped by expert:
+//   gate/up GEMM:  H[r, :] = silu(X[r] Wg_e^T) * (X[r] Wu_e^T)     (K = d, 128 H columns / tile)
+//   down GEMM:     Y[r, :] = H[r] Wd_e^T                           (K = m, 256 Y columns / tile)
+//
+// Persistent kernel: one CTA per SM walks the (M-tile, N-tile) list in M-major order, so the
+// CTAs running at the same time share the weight tiles of the same few experts through L2.
+// Warp 0 issues TMA loads into a STAGES-deep ring of 128-byte-swizzled K-major tiles, warp 1
+// owns TMEM and issues tcgen05.mma (M=128, N=256, K=16) into one of two 256-column fp32
+// accumulators, warps 2..5 drain the other accumulator (one thread per tile row) while the
+// next tile is being multiplied.
+#include "pr2_device.cuh"
+#include "pr2_internal.h"
+
+namespace pr2 {
+namespace {
+
+constexpr int kThreads = 192;
+constexpr int kBK = 64;
+constexpr int kBN = 256;
+constexpr int kStages = 4;
+constexpr int kATile = kTileM * kBK * 2;  // 16 KB
+constexpr int kBTile = kBN * kBK * 2;     // 32 KB
+constexpr int kStageBytes = kATile + kBTile;
+constexpr int kAccCols = kBN;              // one accumulator
+constexpr uint32_t kTmemCols = 2 * kAccCols;
+constexpr int kBarOffset = kStages * kStageBytes;
+constexpr int kSmemBytes = 1024 + kBarOffset + 256;
+
+template <bool kSwiGLU>
+__global__ void __launch_bounds__(kThreads, 1)
+    expert_tc_kernel(const __grid_constant__ CUtensorMap tm_a,
+                     const __grid_constant__ CUtensorMap tm_b0,
+                     const __grid_constant__ CUtensorMap tm_b1, GemmArgs g) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kBarOffset);
+  uint64_t* empty = full + kStages;
+  uint64_t* acc_full = empty + kStages;  // [2]
+  uint64_t* acc_empty = acc_full + 2;    // [2]
+  uint64_t* drain = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  constexpr int kColsPerTile = kSwiGLU ? kBN / 2 : kBN;  // output columns per N-tile
+  const int n_tiles_n = (g.n_out + kColsPerTile - 1) / kColsPerTile;
+  const int num_tiles = (*g.num_tiles) * n_tiles_n;
+  const int KB = g.K / kBK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 4);  // one arrival per epilogue warp
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tm_a);
+    tma_prefetch_desc(&tm_b0);
+    if (kSwiGLU) tma_prefetch_desc(&tm_b1);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tc_fence_before();
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- TMA producer ----------------
+    uint32_t issued = 0, last_par = 0;
+    int stage = 0;
+    uint32_t phase = 0;
+    const uint64_t keep = l2_policy_evict_last();  // expert weights: reused by every M-tile
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+      const int mt = tile / n_tiles_n;
+      const int nt = tile - mt * n_tiles_n;
+      const TileEntry te = g.tiles[mt];
+      const int brow = te.expert * g.b_rows_per_expert + nt * (kSwiGLU ? kBN / 2 : kBN);
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, g.status)) {
+          ok = false;
+          break;
+        }
+        uint8_t* sa = smem + stage * kStageBytes;
+        uint8_t* sb = sa + kATile;
+        mbar_arrive_expect_tx(&full[stage], kStageBytes);
+        tma_load_2d(sa, &tm_a, &full[stage], kb * kBK, te.a_row0);
+        if (kSwiGLU) {
+          tma_load_2d_hint(sb, &tm_b0, &full[stage], kb * kBK, brow, keep);
+          tma_load_2d_hint(sb + kBTile / 2, &tm_b1, &full[stage], kb * kBK, brow, keep);
+        } else {
+          tma_load_2d_hint(sb, &tm_b0, &full[stage], kb * kBK, brow, keep);
+        }
+        issued |= 1u << stage;
+        last_par = (last_par & ~(1u << stage)) | (phase << stage);
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+    for (int s = 0; s < kStages; ++s)
+      if ((issued >> s) & 1u)
+        mbar_wait_slow(&full[s], (last_par >> s) & 1u, nullptr, nullptr, kDrainLimitNs);
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer ----------------
+    constexpr uint32_t idesc = umma_idesc_bf16(kTileM, kBN);
+    int stage = 0;
+    uint32_t phase = 0;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+      if (!mbar_wait(&acc_empty[acc], acc_phase ^ 1u, abort_flag, g.status)) break;
+      tc_fence_after();
+      const uint32_t d_tmem = tmem + acc * kAccCols;
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!mbar_wait(&full[stage], phase, abort_flag, g.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t sa = smem_u32(smem + stage * kStageBytes);
+        const uint32_t sb = sa + kATile;
+#pragma unroll
+        for (int kk = 0; kk < kBK / 16; ++kk)
+          umma_bf16(d_tmem, umma_desc_sw128(sa + kk * 32), umma_desc_sw128(sb + kk * 32), idesc,
+                    (kb > 0 || kk > 0) ? 1u : 0u);
+        umma_commit(&empty[stage]);
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (!ok) break;
+      umma_commit(&acc_full[acc]);
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1u;
+      }
+    }
+    umma_commit(drain);
+    mbar_wait_slow(drain, 0, nullptr, nullptr, kDrainLimitNs);
+  } else if (warp >= 2) {
+    // ---------------- epilogue ----------------
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    __nv_bfloat16* out = static_cast<__nv_bfloat16*>(g.out);
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+      const int mt = tile / n_tiles_n;
+      const int nt = tile - mt * n_tiles_n;
+      const TileEntry te = g.tiles[mt];
+      if (!mbar_wait(&acc_full[acc], acc_phase, abort_flag, g.status)) break;
+      tc_fence_after();
+      const bool live = row < te.rows;
+      __nv_bfloat16* orow = out + static_cast<int64_t>(te.out_row0 + row) * g.n_out;
+      const uint32_t tacc = tmem + acc * kAccCols + (static_cast<uint32_t>(q * 32) << 16);
+      if (kSwiGLU) {
+#pragma unroll 1
+        for (int c0 = 0; c0 < kBN / 2; c0 += 16) {
+          uint32_t rg[16], ru[16];
+          tmem_ld16(tacc + c0, rg);
+          tmem_ld16(tacc + kBN / 2 + c0, ru);
+          tmem_wait_ld(rg);
+          reg_fence(ru);
+          const int col = nt * (kBN / 2) + c0;
+          if (live && col < g.n_out) {
+            uint32_t pk[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float g0 = __uint_as_float(rg[2 * j]), g1 = __uint_as_float(rg[2 * j + 1]);
+              const float u0 = __uint_as_float(ru[2 * j]), u1 = __uint_as_float(ru[2 * j + 1]);
+              const float h0 = __fdividef(g0, 1.0f + __expf(-g0)) * u0;
+              const float h1 = __fdividef(g1, 1.0f + __expf(-g1)) * u1;
+              pk[j] = pack_bf16x2(h0, h1);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(orow + col);
+            dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c0 = 0; c0 < kBN; c0 += 16) {
+          uint32_t rv[16];
+          tmem_ld16(tacc + c0, rv);
+          tmem_wait_ld(rv);
+          const int col = nt * kBN + c0;
+          if (live && col < g.n_out) {
+            uint32_t pk[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              pk[j] = pack_bf16x2(__uint_as_float(rv[2 * j]), __uint_as_float(rv[2 * j + 1]));
+            uint4* dst = reinterpret_cast<uint4*>(orow + col);
+            dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[acc]);
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1u;
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_expert_tc(bool swiglu, const CUtensorMap& tm_a, const CUtensorMap& tm_b0,
+                             const CUtensorMap& tm_b1, const GemmArgs& g, int num_sms,
+                             cudaStream_t st) {
+  if (g.max_tiles <= 0) return cudaSuccess;
+  const int cols = swiglu ? kBN / 2 : kBN;
+  const int64_t bound = static_cast<int64_t>(g.max_tiles) * ((g.n_out + cols - 1) / cols);
+  const int grid = static_cast<int>(bound < num_sms ? bound : num_sms);
+  cudaError_t err;
+  if (swiglu) {
+    err = cudaFuncSetAttribute(expert_tc_kernel<true>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (err != cudaSuccess) return err;
+    expert_tc_kernel<true><<<grid, kThreads, kSmemBytes, st>>>(tm_a, tm_b0, tm_b1, g);
+  } else {
+    err = cudaFuncSetAttribute(expert_tc_kernel<false>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (err != cudaSuccess) return err;
+    expert_tc_kernel<false><<<grid, kThreads, kSmemBytes, st>>>(tm_a, tm_b0, tm_b1, g);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace pr2

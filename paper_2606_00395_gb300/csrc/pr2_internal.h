@@ -1,0 +1,95 @@
+// Host-side interface between the C ABI (api.cu) and the kernel launchers of each .cu file.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/pr2.h"
+
+namespace pr2 {
+
+// One M-tile of a grouped GEMM: rows [a_row0, a_row0 + rows) of the A operand, multiplied by
+// the weights of `expert`, written to rows [out_row0, out_row0 + rows) of the output.
+struct TileEntry {
+  int32_t expert, a_row0, rows, out_row0;
+};
+
+constexpr int kTileM = 128;         // rows per M-tile (one tcgen05 M=128 accumulator)
+constexpr int kDispatchChunk = 256; // flat slots per dispatch block (8 warps x 32 lanes)
+constexpr int kMaxTopK = 8;         // slots kept by the tensor-core routing epilogue
+constexpr int kMaxTopKSimt = 32;    // slots of the fp32 SIMT routing kernel
+constexpr int kMaxExperts = 256;    // routed experts supported by the routing kernels
+constexpr int kMaxExpertsDispatch = 1024;
+
+// ---- routing (route_simt.cu, route_tc.cu) -------------------------------------------------
+cudaError_t launch_route_simt(const pr2_dims& dm, bool predict, const float* h, const float* W,
+                              const float* Wp, const int32_t* idx_in, int32_t* idx_out,
+                              float* gates, float* logits_or_probs, int64_t* near_tie,
+                              int32_t* status, cudaStream_t st);
+
+struct RouteTcArgs {
+  int T, d, N, k;
+  const int32_t* idx_in;   // replay: cached route
+  int32_t* idx_out;        // predict: route out
+  float* gates;
+  float* logits_or_probs;  // predict: p_old [T,N]; replay: rho [T,N]; nullable
+  int64_t* near_tie;
+  int32_t* status;
+};
+cudaError_t launch_route_tc(bool predict, const CUtensorMap& tm_h, const CUtensorMap& tm_w,
+                            const CUtensorMap& tm_wp, const RouteTcArgs& a, cudaStream_t st);
+
+// ---- dispatch and combine (dispatch.cu) ----------------------------------------------------
+struct DispatchArgs {
+  const int32_t* idx;
+  int64_t T;
+  int k, N, d, esz, n_shared;
+  int32_t* blk_hist;     // [nblk, N] block histograms, scanned in place into block bases
+  int32_t* counts;       // [N]
+  int32_t* offsets;      // [N+1]
+  int32_t* perm;         // [T*k]
+  int32_t* inv;          // [T*k]
+  TileEntry* tiles;      // [max_mtiles]
+  int32_t* num_tiles;    // [2]: routed M-tiles, shared M-tiles
+  TileEntry* stiles1;    // [n_shared * ceil(T/128)] gate/up GEMM of the shared experts
+  TileEntry* stiles2;    // same, down GEMM
+  const void* h;
+  void* xperm;           // [T*k, d]
+  int32_t* status;
+};
+cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st);
+
+struct CombineArgs {
+  const void* Y;        // [T*k, d] expert outputs in dispatch order
+  const void* Ys;       // [n_shared, T, d] shared-expert outputs (nullable)
+  const int32_t* inv;   // [T*k]
+  const float* gates;   // [T*k]
+  int64_t T;
+  int k, d, n_shared, bf16;
+  void* out;            // [T, d]
+};
+cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st);
+
+// ---- grouped expert GEMMs (expert_tc.cu, expert_simt.cu) -----------------------------------
+struct GemmArgs {
+  const TileEntry* tiles;
+  const int32_t* num_tiles;  // device count of valid entries in `tiles`
+  int max_tiles;             // host bound on that count
+  int K;                     // reduction length
+  int n_out;                 // output columns
+  int b_rows_per_expert;     // rows of one expert's weight matrix (m for gate/up, d for down)
+  void* out;                 // [rows, n_out]
+  int32_t* status;
+};
+// swiglu: out = silu(A Wg^T) * (A Wu^T) (tm_b0 = gate, tm_b1 = up); else out = A Wb^T.
+cudaError_t launch_expert_tc(bool swiglu, const CUtensorMap& tm_a, const CUtensorMap& tm_b0,
+                             const CUtensorMap& tm_b1, const GemmArgs& g, int num_sms,
+                             cudaStream_t st);
+cudaError_t launch_expert_simt(bool swiglu, const float* A, const float* Wb0, const float* Wb1,
+                               const GemmArgs& g, cudaStream_t st);
+
+// ---- self test (api.cu) --------------------------------------------------------------------
+cudaError_t launch_wait_selftest(int32_t* status, int64_t timeout_ns, cudaStream_t st);
+
+}  // namespace pr2

@@ -1,0 +1,110 @@
+"""The C-ABI library on the CPU: it builds, loads, exports every symbol include/pr2.h declares,
+and rejects invalid arguments on the host before any CUDA call (no GPU needed)."""
+import ctypes
+
+import pytest
+
+from paper_2606_00395_gb300 import binding as B
+from paper_2606_00395_gb300 import build
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return B.load()
+
+
+def test_exports_every_declared_symbol(lib):
+    names = B.declared_symbols()
+    assert {"pr2_route_predict", "pr2_route_replay", "pr2_moe_forward", "pr2_moe_workspace_bytes",
+            "pr2_strerror"} <= set(names)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_strerror_names_every_code(lib):
+    for code in range(7):
+        assert B.pr2_strerror(code) and B.pr2_strerror(code) != "unknown status"
+    assert B.pr2_strerror(99) == "unknown status"
+
+
+def test_workspace_bytes_grow_with_the_layer(lib):
+    small = B.pr2_moe_workspace_bytes(B.dims(256, 2048, 128, 8, 768))
+    big = B.pr2_moe_workspace_bytes(B.dims(4096, 2048, 128, 8, 768))
+    shared = B.pr2_moe_workspace_bytes(B.dims(4096, 2048, 128, 8, 768, n_shared=1))
+    assert 0 < small < big < shared
+    # dominated by the permuted rows, the expert hidden activations and the expert outputs
+    F = 4096 * 8
+    assert big >= 2 * F * (2048 + 768 + 2048)
+
+
+@pytest.mark.parametrize("bad", [
+    dict(T=-1), dict(d=0), dict(N=0), dict(k=0), dict(k=129), dict(m=0), dict(n_shared=-1),
+])
+def test_invalid_dims_are_rejected(lib, bad):
+    kw = dict(T=64, d=2048, N=128, k=8, m=768)
+    kw.update(bad)
+    dm = B.dims(**kw)
+    assert B.pr2_moe_workspace_bytes(dm) == 0
+    fake = ctypes.c_void_p(256)
+    code = lib.pr2_route_predict(ctypes.byref(dm), fake, fake, fake, fake, fake, None, None, None,
+                                 None)
+    assert code == 1
+
+
+@pytest.mark.parametrize("kw", [
+    dict(d=2000),          # bf16 needs d % 64 == 0
+    dict(m=700),           # bf16 needs m % 64 == 0
+    dict(N=100, k=8),      # bf16 needs N % 16 == 0
+    dict(k=9),             # bf16 routing keeps at most 8 slots
+    dict(N=512, k=8),      # at most 256 routed experts
+])
+def test_unsupported_shapes_are_rejected(lib, kw):
+    base = dict(T=64, d=2048, N=128, k=8, m=768)
+    base.update(kw)
+    dm = B.dims(**base)
+    fake = ctypes.c_void_p(256)
+    assert lib.pr2_route_predict(ctypes.byref(dm), fake, fake, fake, fake, fake, None, None, None,
+                                 None) == 2
+
+
+def test_null_pointers_and_short_workspace_are_rejected(lib):
+    dm = B.dims(64, 2048, 128, 8, 768)
+    fake = ctypes.c_void_p(256)
+    P = [fake] * 6
+    assert lib.pr2_route_predict(ctypes.byref(dm), None, *P[:4], None, None, None, None) == 1
+    assert lib.pr2_route_replay(ctypes.byref(dm), fake, fake, None, fake, None, None, None) == 1
+    # misaligned device pointer
+    odd = ctypes.c_void_p(258)
+    assert lib.pr2_route_predict(ctypes.byref(dm), odd, *P[:4], None, None, None, None) == 1
+    ws = B.pr2_moe_workspace_bytes(dm)
+    args = [ctypes.byref(dm), fake, fake, fake, fake, fake, fake, None, None, None, fake, None,
+            None]
+    assert lib.pr2_moe_forward(*args, fake, ctypes.c_size_t(ws - 1), None, None, None) == 6
+    assert lib.pr2_moe_forward(*args, None, ctypes.c_size_t(ws), None, None, None) == 6
+    assert lib.pr2_moe_forward(*args, ctypes.c_void_p(512 + 16), ctypes.c_size_t(ws), None,
+                               None, None) == 6
+    # shared-expert weights must be given iff n_shared > 0
+    dm1 = B.dims(64, 2048, 128, 8, 768, n_shared=1)
+    args1 = [ctypes.byref(dm1), fake, fake, fake, fake, fake, fake, None, None, None, fake, None,
+             None]
+    assert lib.pr2_moe_forward(*args1, fake, ctypes.c_size_t(1 << 40), None, None, None) == 1
+    # sync-status needs a status word
+    dms = B.dims(64, 2048, 128, 8, 768, flags=B.PR2_F_SYNC_STATUS)
+    assert lib.pr2_route_predict(ctypes.byref(dms), *P[:5], None, None, None, None) == 1
+
+
+def test_empty_layer_is_a_no_op(lib):
+    dm = B.dims(0, 2048, 128, 8, 768)
+    assert lib.pr2_route_predict(ctypes.byref(dm), None, None, None, None, None, None, None,
+                                 None, None) == 0
+    ws = B.pr2_moe_workspace_bytes(dm)
+    assert ws > 0
+    assert lib.pr2_moe_forward(ctypes.byref(dm), *([None] * 12), None, ctypes.c_size_t(0), None,
+                               None, None) == 0
+
+
+def test_selftest_rejects_out_of_range_limits(lib):
+    assert lib.pr2_selftest_wait_timeout(None, 1000, None) == 1
+    assert lib.pr2_selftest_wait_timeout(ctypes.c_void_p(256), 10, None) == 1
+    assert lib.pr2_selftest_wait_timeout(ctypes.c_void_p(256), 10 ** 10, None) == 1

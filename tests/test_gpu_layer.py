@@ -1,0 +1,158 @@
+"""GPU parity: every step of the layer through the C ABI against the CPU oracle.
+
+Small layers are compared element by element in full (several M-tiles per expert, ragged
+tails, partial N-tiles); the full-size workloads are compared on all routes and permutations
+and on a seeded sample of layer outputs.  Tolerances are defined in ``layer_harness``."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_00395_gb300 import binding as B
+from paper_2606_00395_gb300 import synth
+from tests import layer_harness as H
+
+pytestmark = pytest.mark.gpu
+
+SMALL = {
+    # fp32 SIMT path, the tiny workload exactly
+    "tiny_fp32": synth.CONFIGS["tiny_fp32"],
+    # bf16, ~175 rows per expert -> 2 M-tiles per expert, 2 gate/up N-tiles, ragged T
+    "bf16_multitile": synth.LayerConfig("bf16_multitile", T=700, d=256, N=16, k=4, m=256),
+    # bf16, partial N-tiles in both GEMMs (m = 192 = 128 + 64, d = 320 = 256 + 64), k = 6
+    "bf16_partial_n": synth.LayerConfig("bf16_partial_n", T=333, d=320, N=32, k=6, m=192),
+    # bf16 with a shared expert, N = 256 routed experts (two 256-column MMAs in routing)
+    "bf16_shared_n256": synth.LayerConfig("bf16_shared_n256", T=200, d=128, N=256, k=8, m=128,
+                                          n_shared=1),
+}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_00395_gb300 import build
+    build.build()
+    B.load()
+
+
+def _full_layer_check(cfg, seed=0):
+    L = synth.make_layer(cfg, seed=seed)
+    Ld = H.to_dev(L)
+    W2 = synth.make_drifted_router(L["W_router"], seed=seed)
+    # ---- rollout: route prediction (Eqs. pr2_predict, pr2_route)
+    g = H.gpu_predict(cfg, Ld)
+    orc = oracle.route_predict(L["x"], L["W_router"], L["W_pred"], cfg.k)
+    exempt = H.check_routes(orc, H.cpu(g["idx"]).numpy())
+    gidx = H.cpu(g["idx"]).numpy()
+    H.rowwise_close(H.cpu(g["gates"]).numpy(), np.take_along_axis(orc["probs"], gidx, 1))
+    H.rowwise_close(H.cpu(g["logits"]).numpy(), orc["logits"])
+    assert int(g["status"].item()) == 0
+    # ---- replay of the oracle's recorded route with the drifted router (Sec. 4.1)
+    idx_rec = torch.from_numpy(orc["idx"]).cuda()
+    r = H.gpu_replay(cfg, Ld, W2.cuda(), idx_rec)
+    orep = oracle.route_replay(L["x"], W2, orc["idx"])
+    H.rowwise_close(H.cpu(r["gates"]).numpy(), orep["gates"])
+    H.rowwise_close(H.cpu(r["probs"]).numpy(), orep["probs"])
+    assert int(r["status"].item()) == 0
+    # ---- layer output on the recorded route with replay gates (Eq. pr2_output)
+    gates_rep = torch.from_numpy(orep["gates"].astype(np.float32)).cuda()
+    f = H.gpu_forward(cfg, Ld, idx_rec, gates_rep)
+    assert f["code"] == 0 and int(f["status"].item()) == 0
+    operm = oracle.permute(orc["idx"], cfg.N)
+    assert np.array_equal(H.cpu(f["counts"]).numpy(), operm["counts"])
+    nvalid = int(operm["offsets"][-1])
+    assert np.array_equal(H.cpu(f["perm"]).numpy()[:nvalid], operm["perm"])
+    want = oracle.moe_forward(L["x"], orc["idx"], orep["gates"], L["W_gate"], L["W_up"],
+                              L["W_down"], L["Ws_gate"], L["Ws_up"], L["Ws_down"])
+    err = H.normwise_close(H.cpu(f["out"]).float().numpy(), want, H.OUT_TOL[cfg.dtype])
+    # ---- rollout layer output on the GPU's own route (Eq. pr2_old_output), non-tie tokens
+    f2 = H.gpu_forward(cfg, Ld, g["idx"], g["gates"])
+    want2 = oracle.moe_forward(L["x"], orc["idx"], orc["gates"], L["W_gate"], L["W_up"],
+                               L["W_down"], L["Ws_gate"], L["Ws_up"], L["Ws_down"])
+    keep = orc["margin"] >= H.TIE_GAP
+    H.normwise_close(H.cpu(f2["out"]).float().numpy()[keep], want2[keep], H.OUT_TOL[cfg.dtype])
+    return exempt, err
+
+
+@pytest.mark.parametrize("name", list(SMALL))
+def test_small_layer_matches_oracle_everywhere(name):
+    exempt, err = _full_layer_check(SMALL[name])
+    print(f"{name}: near-tie tokens {exempt}, output error {err:.2e}")
+
+
+def test_near_tie_counter_tracks_the_oracle_margin():
+    cfg = synth.LayerConfig("q300", T=300, d=2048, N=128, k=8, m=768)
+    L = synth.make_layer(cfg)
+    Ld = H.to_dev(L)
+    g = H.gpu_predict(cfg, Ld)
+    orc = oracle.route_predict(L["x"], L["W_router"], L["W_pred"], cfg.k)
+    H.check_routes(orc, H.cpu(g["idx"]).numpy())
+    n_orc = int(np.sum(orc["margin"] < H.TIE_GAP))
+    n_gpu = int(g["near_tie"].item())
+    # the GPU classifies with its own fp32 probabilities: allow tokens right at the threshold
+    borderline = int(np.sum(np.abs(orc["margin"] - H.TIE_GAP) < 2e-6))
+    assert abs(n_gpu - n_orc) <= borderline, (n_gpu, n_orc, borderline)
+
+
+def test_zero_predictor_replay_reproduces_rollout():
+    """W_p = 0 and the same router: replaying the recorded route gives the rollout gates and
+    the same layer output (routing replay, R2, is Pr^2 with a zero predictor)."""
+    cfg = synth.LayerConfig("r2", T=260, d=512, N=64, k=8, m=256)
+    L = synth.make_layer(cfg, seed=5)
+    L["W_pred"] = torch.zeros_like(L["W_pred"])
+    Ld = H.to_dev(L)
+    g = H.gpu_predict(cfg, Ld)
+    r = H.gpu_replay(cfg, Ld, Ld["W_router"], g["idx"])
+    gg, rg = H.cpu(g["gates"]), H.cpu(r["gates"])
+    assert torch.max(torch.abs(gg - rg)).item() <= 1e-6
+    o1 = H.gpu_forward(cfg, Ld, g["idx"], g["gates"])["out"]
+    o2 = H.gpu_forward(cfg, Ld, g["idx"], r["gates"])["out"]
+    H.normwise_close(H.cpu(o2).float().numpy(), H.cpu(o1).float().numpy(), 1e-2)
+    print("bit-exact replay gates:", torch.equal(gg, rg))
+
+
+def test_layer_is_deterministic():
+    cfg = synth.LayerConfig("det", T=1000, d=512, N=32, k=8, m=256)
+    L = synth.make_layer(cfg, seed=11)
+    Ld = H.to_dev(L)
+    g = H.gpu_predict(cfg, Ld)
+    a = H.gpu_forward(cfg, Ld, g["idx"], g["gates"])
+    b = H.gpu_forward(cfg, Ld, g["idx"], g["gates"])
+    assert torch.equal(a["out"], b["out"]) and torch.equal(a["perm"], b["perm"])
+
+
+def test_invalid_replay_indices_are_flagged_and_skipped():
+    cfg = synth.LayerConfig("bad", T=130, d=256, N=16, k=4, m=128)
+    L = synth.make_layer(cfg, seed=2)
+    Ld = H.to_dev(L)
+    orc = oracle.route_predict(L["x"], L["W_router"], L["W_pred"], cfg.k)
+    idx = orc["idx"].copy()
+    idx[3, 1] = 16       # out of range
+    idx[7, 2] = -5       # negative
+    idx[129, 3] = idx[129, 0]  # duplicate within the token (last, ragged tile)
+    idx_d = torch.from_numpy(idx).cuda()
+    r = H.gpu_replay(cfg, Ld, Ld["W_router"], idx_d)
+    orep = oracle.route_replay(L["x"], L["W_router"], idx)
+    assert orep["bad"] == 3
+    rg = H.cpu(r["gates"]).numpy()
+    assert rg[3, 1] == 0 and rg[7, 2] == 0 and rg[129, 3] == 0
+    H.rowwise_close(rg, orep["gates"])
+    assert int(r["status"].item()) & B.PR2_STATUS_BAD_INDEX
+    f = H.gpu_forward(cfg, Ld, idx_d, r["gates"])
+    assert int(f["status"].item()) & B.PR2_STATUS_BAD_INDEX
+    operm = oracle.permute(idx, cfg.N)
+    assert np.array_equal(H.cpu(f["counts"]).numpy(), operm["counts"])
+    assert np.array_equal(H.cpu(f["perm"]).numpy()[: operm["perm"].size], operm["perm"])
+    want = oracle.moe_forward(L["x"], idx, orep["gates"], L["W_gate"], L["W_up"], L["W_down"])
+    H.normwise_close(H.cpu(f["out"]).float().numpy(), want, H.OUT_TOL["bf16"])
+    # with PR2_F_SYNC_STATUS the call itself reports the bad index
+    f3 = H.gpu_forward(cfg, Ld, idx_d, r["gates"], flags=B.PR2_F_SYNC_STATUS)
+    assert f3["code"] == 4
+
+
+def test_bounded_wait_reports_timeout_instead_of_hanging():
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    assert B.pr2_selftest_wait_timeout(status, 20_000_000) == 0
+    torch.cuda.synchronize()
+    assert int(status.item()) == B.PR2_STATUS_TIMEOUT
