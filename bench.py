@@ -1,0 +1,403 @@
+#!/usr/bin/env python
+"""Throughput of the Pr^2 MoE layer forward (rollout predict-route + training replay) on GB300.
+
+One step = the whole hot path over one batch of T tokens in both modes:
+  rollout:  pr2_route_predict (router + predictor GEMM, softmax, top-k, route record)
+            -> pr2_moe_forward (dispatch, grouped gate/up + SwiGLU GEMM, down GEMM, combine)
+  replay:   pr2_route_replay on the recorded route with the drifted current router
+            -> pr2_moe_forward with the replay gates.
+value = tokens/s = T * ranks / (max over ranks of the summed per-step device time).
+L2 is flushed (512 MiB write) before every step; the flush is outside the timed intervals.
+
+--impl reference times the CPU oracle (the reference of this build) on a bounded token sample of
+the same workload, on the host cores, and prints the same JSON line with "impl": "reference".
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2606_00395_gb300 import binding as B  # noqa: E402
+from paper_2606_00395_gb300 import cost, synth  # noqa: E402
+
+METRIC = "MoE-layer tokens/s (predict-route & replay fwd) on 1 GB300; % of roofline"
+FLUSH_BYTES = 512 << 20
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["pr2", "reference"], default="pr2")
+    ap.add_argument("--workload", default="qwen3_30b_a3b", choices=sorted(synth.CONFIGS))
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        p = json.load(open(path))
+        return dict(hbm=float(p["hbm_gbs"]), bf16=float(p["bf16_tflops"]),
+                    bf16_sustained=float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
+
+
+def workload_desc(cfg):
+    return dict(workload=cfg.name, T=cfg.T, d=cfg.d, N=cfg.N, k=cfg.k, m=cfg.m,
+                n_shared=cfg.n_shared, modes="rollout+replay", tokens_per_step=cfg.T,
+                weights="N(0,0.02) seed 0, replay router drift N(0,0.002) seed 1",
+                l2="flushed before every step (512 MiB write), flush not timed",
+                parallelism="replicas")
+
+
+# ----------------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+        uuid = str(getattr(torch.cuda.get_device_properties(index), "uuid", index))
+        sel = uuid if uuid.startswith("GPU-") else (f"GPU-{uuid}" if "-" in uuid else str(index))
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", sel, f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.fh,
+                stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.fh.close()
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                rows.append((float(parts[0]), float(parts[1]), parts[3:7]))
+            except ValueError:
+                continue
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, fl in rows for i, v in enumerate(fl)
+                          if v.lower() == "active"})
+        return dict(sm_mhz=statistics.median(r[0] for r in rows), sm_max_mhz=max(r[1] for r in rows),
+                    reasons=reasons, samples=len(rows))
+
+
+# ----------------------------------------------------------------------------------- oracle
+
+def oracle_layer_seconds(cfg, Lh, W2h, toks):
+    """Run the CPU oracle over `toks` in both modes (rollout + replay); return seconds."""
+    import oracle
+    x = Lh["x"][torch.from_numpy(toks)]
+    t0 = time.perf_counter()
+    r = oracle.route_predict(x, Lh["W_router"], Lh["W_pred"], cfg.k)
+    oracle.moe_forward(x, r["idx"], r["gates"], Lh["W_gate"], Lh["W_up"], Lh["W_down"],
+                       Lh["Ws_gate"], Lh["Ws_up"], Lh["Ws_down"])
+    rep = oracle.route_replay(x, W2h, r["idx"])
+    oracle.moe_forward(x, r["idx"], rep["gates"], Lh["W_gate"], Lh["W_up"], Lh["W_down"],
+                       Lh["Ws_gate"], Lh["Ws_up"], Lh["Ws_down"])
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(cfg, Lh, W2h, target_s):
+    """Time the oracle on a growing token sample until ~target_s seconds of CPU work."""
+    import oracle
+    n, spent, toks_done = 8, 0.0, 0
+    while True:
+        toks = synth.make_token_sample(cfg.T, n, 7 + n).numpy()
+        dt = oracle_layer_seconds(cfg, Lh, W2h, toks)
+        spent, toks_done = dt, len(toks)
+        if dt * 2 > target_s or n >= cfg.T:
+            break
+        n = min(cfg.T, n * 2)
+    return dict(value=toks_done / spent, unit="tokens/s", cores=oracle.num_threads(),
+                kind="oracle",
+                sample=f"{toks_done} seeded tokens of {cfg.name} through both modes "
+                       f"(route predict + layer, route replay + layer), fp64, {spent:.1f} s")
+
+
+def host_layer(cfg, L):
+    return {k: (v.cpu() if v is not None else None) for k, v in L.items()}
+
+
+# ----------------------------------------------------------------------------------- pr2 arm
+
+def run_pr2(args, rank, world, local_rank):
+    torch.cuda.set_device(local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    cfg = synth.CONFIGS[args.workload]
+    dev = "cuda"
+    L = synth.make_layer(cfg, seed=0, device=dev)
+    W2 = synth.make_drifted_router(L["W_router"])
+    dm = B.dims(cfg.T, cfg.d, cfg.N, cfg.k, cfg.m, cfg.n_shared, cfg.dtype)
+    ws = B.alloc_workspace(dm)
+    idx, gates, logits = B.alloc_route(dm, logits=True)
+    rgates = torch.empty_like(gates)
+    out1 = torch.empty(cfg.T, cfg.d, dtype=cfg.torch_dtype, device=dev)
+    out2 = torch.empty_like(out1)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    near = torch.zeros(1, dtype=torch.int64, device=dev)
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def ev():
+        e = torch.cuda.Event(enable_timing=True)
+        e.record()  # creates the underlying cudaEvent_t
+        return e
+
+    def step(x, evs):
+        evs[0].record()
+        B.check(B.pr2_route_predict(dm, x, L["W_router"], L["W_pred"], idx, gates, logits, near,
+                                    status), "pr2_route_predict")
+        evs[1].record()
+        B.check(B.pr2_moe_forward(dm, x, idx, gates, L["W_gate"], L["W_up"], L["W_down"],
+                                  L["Ws_gate"], L["Ws_up"], L["Ws_down"], out1, workspace=ws,
+                                  status=status, events=evs[2]), "pr2_moe_forward")
+        evs[3].record()
+        B.check(B.pr2_route_replay(dm, x, W2, idx, rgates, None, status), "pr2_route_replay")
+        evs[4].record()
+        B.check(B.pr2_moe_forward(dm, x, idx, rgates, L["W_gate"], L["W_up"], L["W_down"],
+                                  L["Ws_gate"], L["Ws_up"], L["Ws_down"], out2, workspace=ws,
+                                  status=status, events=evs[5]), "pr2_moe_forward")
+        evs[6].record()
+
+    def make_evs():
+        a = [ev() for _ in range(5)]
+        b = [ev() for _ in range(5)]
+        return [ev(), ev(), (B.stage_events(a), a), ev(), ev(), (B.stage_events(b), b), ev()]
+
+    def run(n, evsets, x=None):
+        for i in range(n):
+            flush.fill_(i & 0xFF)
+            e = evsets[i]
+            step(L["x"] if x is None else x,
+                 [e[0], e[1], e[2][0], e[3], e[4], e[5][0], e[6]])
+
+    # warm-up
+    wev = [make_evs() for _ in range(args.warmup)]
+    run(args.warmup, wev)
+    torch.cuda.synchronize()
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())} after warm-up")
+    evsets = [make_evs() for _ in range(args.steps)]
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(torch.cuda.current_device())
+    time.sleep(0.3)
+    near.zero_()
+    run(args.steps, evsets)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    near_per_step = int(near.item()) / args.steps
+    if dist is not None:
+        dist.barrier()
+
+    def el(a, b):
+        return a.elapsed_time(b)  # ms
+
+    per = dict(step=[], route_predict=[], route_replay=[], dispatch=[], gate_up=[], down=[],
+               combine=[], layer_rollout=[], layer_replay=[])
+    for e in evsets:
+        per["step"].append(el(e[0], e[6]))
+        per["route_predict"].append(el(e[0], e[1]))
+        per["route_replay"].append(el(e[3], e[4]))
+        per["layer_rollout"].append(el(e[0], e[3]))
+        per["layer_replay"].append(el(e[3], e[6]))
+        for _, st in (e[2], e[5]):
+            per["dispatch"].append(el(st[0], st[1]))
+            per["gate_up"].append(el(st[1], st[2]))
+            per["down"].append(el(st[2], st[3]))
+            per["combine"].append(el(st[3], st[4]))
+    total_ms = sum(per["step"])
+    if dist is not None:
+        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    value = cfg.T * world * args.steps / (total_ms / 1e3)
+    mean = {k: statistics.mean(v) for k, v in per.items()}
+
+    # ---- per-kernel roofline (algorithmic work / measured duration)
+    pk = peaks()
+    F = cfg.T * cfg.k
+    counts = torch.empty(cfg.N, dtype=torch.int32, device=dev)
+    B.check(B.pr2_moe_forward(dm, L["x"], idx, gates, L["W_gate"], L["W_up"], L["W_down"],
+                              L["Ws_gate"], L["Ws_up"], L["Ws_down"], out1, counts=counts,
+                              workspace=ws, status=status), "pr2_moe_forward")
+    hit = int((counts > 0).sum().item())
+    work = {
+        "route_predict": cost.route_predict_work(cfg.T, cfg.d, cfg.N, cfg.k, cfg.dtype, True),
+        "route_replay": cost.route_replay_work(cfg.T, cfg.d, cfg.N, cfg.k, cfg.dtype, False),
+        "dispatch": cost.dispatch_work(cfg.T, cfg.d, cfg.k, cfg.dtype),
+        "gate_up": cost.expert_gate_up_work(F, cfg.d, cfg.m, hit, cfg.dtype),
+        "down": cost.expert_down_work(F, cfg.d, cfg.m, hit, cfg.dtype),
+        "combine": cost.combine_work(cfg.T, cfg.d, cfg.k, cfg.n_shared, cfg.dtype),
+    }
+    if cfg.n_shared:
+        sg = cost.expert_gate_up_work(cfg.T * cfg.n_shared, cfg.d, cfg.m, cfg.n_shared, cfg.dtype)
+        sd = cost.expert_down_work(cfg.T * cfg.n_shared, cfg.d, cfg.m, cfg.n_shared, cfg.dtype)
+        work["gate_up"] = cost.KernelWork(work["gate_up"].bytes + sg.bytes,
+                                          work["gate_up"].flops + sg.flops)
+        work["down"] = cost.KernelWork(work["down"].bytes + sd.bytes, work["down"].flops + sd.flops)
+    kernels = {}
+    for name, w in work.items():
+        ms = mean[name]
+        t_hbm = w.bytes / (pk["hbm"] * 1e9) * 1e3
+        t_tc = w.flops / (pk["bf16"] * 1e12) * 1e3
+        if t_tc > t_hbm:
+            kernels[name] = dict(ms=ms, bound="tensor", achieved=w.flops / (ms * 1e-3) / 1e12,
+                                 peak=pk["bf16"], unit="TFLOP/s", frac=t_tc / ms,
+                                 algorithmic_flops=w.flops, algorithmic_bytes=w.bytes)
+        else:
+            kernels[name] = dict(ms=ms, bound="hbm", achieved=w.bytes / (ms * 1e-3) / 1e9,
+                                 peak=pk["hbm"], unit="GB/s", frac=t_hbm / ms,
+                                 algorithmic_flops=w.flops, algorithmic_bytes=w.bytes)
+    dom = max(("gate_up", "down"), key=lambda n: kernels[n]["ms"])
+    dk = kernels[dom]
+    roofline = dict(kernel=f"expert_tc_kernel ({dom})", bound=dk["bound"], achieved=dk["achieved"],
+                    peak=dk["peak"], unit=dk["unit"], frac=dk["frac"], traffic=None,
+                    peak_source=f"{pk['source']} (MEASURED_PEAKS.json burst)"
+                    if pk["source"] == "measured" else "fallback",
+                    algorithmic=("flops" if dk["bound"] == "tensor" else "bytes"),
+                    per_launch_units=f"{F} token-expert rows x (d={cfg.d}, m={cfg.m})")
+
+    # ---- end to end through the public API with host buffers
+    xh = torch.empty(cfg.T, cfg.d, dtype=cfg.torch_dtype, pin_memory=True)
+    xh.copy_(L["x"].cpu())
+    out1h = torch.empty(cfg.T, cfg.d, dtype=cfg.torch_dtype, pin_memory=True)
+    out2h = torch.empty_like(out1h)
+    idxh = torch.empty(cfg.T, cfg.k, dtype=torch.int32, pin_memory=True)
+    xd = torch.empty_like(L["x"])
+    e2e_ms = []
+    for i in range(args.warmup + args.steps):
+        flush.fill_(i & 0xFF)
+        a = ev()
+        xd.copy_(xh, non_blocking=True)
+        e = make_evs()
+        step(xd, [e[0], e[1], e[2][0], e[3], e[4], e[5][0], e[6]])
+        out1h.copy_(out1, non_blocking=True)
+        out2h.copy_(out2, non_blocking=True)
+        idxh.copy_(idx, non_blocking=True)
+        b = ev()
+        b.synchronize()
+        if i >= args.warmup:
+            e2e_ms.append(a.elapsed_time(b))
+    e2e_total = sum(e2e_ms)
+    if dist is not None:
+        t = torch.tensor([e2e_total], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_total = float(t.item())
+    esz = 2 if cfg.dtype == "bf16" else 4
+    e2e = dict(value=cfg.T * world * args.steps / (e2e_total / 1e3), unit="tokens/s",
+               h2d_bytes_per_step=cfg.T * cfg.d * esz,
+               d2h_bytes_per_step=2 * cfg.T * cfg.d * esz + cfg.T * cfg.k * 4)
+
+    launches_per_step = 2 + 2 * (7 + (2 if cfg.n_shared else 0))
+    line = dict(metric=METRIC, value=value, unit="tokens/s", n_gpus=world, steps=args.steps,
+                warmup=args.warmup, ms_per_step=total_ms / args.steps, higher_is_better=True,
+                scaling="weak", vs_baseline=None, dtype=cfg.dtype, data="synthetic",
+                config=workload_desc(cfg), roofline=roofline, e2e=e2e,
+                gpu_launches=launches_per_step * args.steps, clocks=clk,
+                modes=dict(rollout_tokens_per_s=cfg.T / (mean["layer_rollout"] / 1e3),
+                           replay_tokens_per_s=cfg.T / (mean["layer_replay"] / 1e3)),
+                kernels=kernels, near_tie_tokens_per_step=near_per_step)
+
+    if rank == 0 and not args.no_cpu_baseline:
+        Lh = host_layer(cfg, L)
+        line["cpu_baseline"] = cpu_baseline(cfg, Lh, W2.cpu(), args.cpu_seconds)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------------- reference
+
+def run_reference(args, rank):
+    if rank != 0:
+        return
+    import oracle
+    cfg = synth.CONFIGS[args.workload]
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    L = synth.make_layer(cfg, seed=0, device=dev)
+    W2 = synth.make_drifted_router(L["W_router"]).cpu()
+    Lh = host_layer(cfg, L)
+    del L
+    n_tok = 8
+    times = []
+    for i in range(args.warmup + args.steps):
+        toks = synth.make_token_sample(cfg.T, n_tok, 100 + i).numpy()
+        dt = oracle_layer_seconds(cfg, Lh, W2, toks)
+        if i >= args.warmup:
+            times.append(dt)
+    total = sum(times)
+    value = n_tok * args.steps / total
+    line = dict(metric=METRIC, value=value, unit="tokens/s", n_gpus=1, steps=args.steps,
+                warmup=args.warmup, ms_per_step=1e3 * total / args.steps, higher_is_better=True,
+                scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
+                config=workload_desc(cfg), impl="reference",
+                cpu_baseline=dict(value=value, unit="tokens/s", cores=oracle.num_threads(),
+                                  kind="oracle",
+                                  sample=f"{n_tok} seeded tokens of {cfg.name} per step, both "
+                                         f"modes, fp64 CPU oracle"),
+                e2e=dict(value=value, unit="tokens/s", h2d_bytes_per_step=0,
+                         d2h_bytes_per_step=0))
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank)
+        return
+    from paper_2606_00395_gb300 import build
+    if local_rank == 0:
+        build.build()
+    else:
+        t0 = time.time()
+        while not build.up_to_date() and time.time() - t0 < 600:
+            time.sleep(1.0)
+    run_pr2(args, rank, world, local_rank)
+
+
+if __name__ == "__main__":
+    main()
