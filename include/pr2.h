@@ -138,6 +138,33 @@ pr2_status pr2_moe_forward(const pr2_dims* dims, const void* h, const int32_t* i
                            void* workspace, size_t ws_bytes, int32_t* status_dev,
                            const pr2_stage_events* events, void* stream);
 
+/*
+ * pr2_moe_forward without a caller-provided workspace.  The paper has no counterpart: this
+ * entry point exists for callers that cannot allocate device memory where they run the layer
+ * (a runtime whose pool owns all device memory, a hot path on which cudaMalloc/cudaFree and
+ * their device-wide synchronisation are not allowed, a plug-in with a fixed memory budget).
+ * Same arguments and results as pr2_moe_forward minus workspace/ws_bytes/events; the scratch
+ * is one array of pr2_static_scratch_bytes() bytes (32 MiB) compiled into the library, which
+ * every GPU that loads the library keeps reserved until the process exits.  The call allocates
+ * nothing.
+ *  - Layers whose pr2_moe_workspace_bytes(dims) exceeds pr2_static_scratch_bytes() are
+ *    rejected with PR2_ERR_WORKSPACE before anything is launched (e.g. the Qwen3-shaped layer
+ *    up to ~400 tokens fits; a 4096-token batch does not).
+ *  - The first call on a device looks up the array's device address (cudaGetSymbolAddress,
+ *    with that device current); make that first call before any stream capture.
+ *  - All calls on a device share the one array: calls whose kernels overlap on the GPU (other
+ *    streams, other host threads) race on it and corrupt each other's results.  Serialise them,
+ *    e.g. by issuing them on one stream.
+ */
+pr2_status pr2_moe_forward_static(const pr2_dims* dims, const void* h, const int32_t* idx,
+                                  const float* gates, const void* W_gate, const void* W_up,
+                                  const void* W_down, const void* Ws_gate, const void* Ws_up,
+                                  const void* Ws_down, void* out, int32_t* counts,
+                                  int32_t* perm, int32_t* status_dev, void* stream);
+
+/* Size in bytes of the scratch array used by pr2_moe_forward_static (no paper counterpart). */
+size_t pr2_static_scratch_bytes(void);
+
 /* Static, human-readable name of a status code. */
 const char* pr2_strerror(pr2_status s);
 

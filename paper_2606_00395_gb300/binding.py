@@ -175,3 +175,37 @@ def alloc_route(dm: Dims, device="cuda", logits: bool = False):
     gates = torch.empty(T, k, dtype=torch.float32, device=device)
     aux = torch.empty(T, N, dtype=torch.float32, device=device) if logits else None
     return idx, gates, aux
+
+
+# ---- workspace-free layer forward (for callers that cannot allocate device memory) -----------
+
+_static_ready = False
+
+
+def _static_lib() -> ctypes.CDLL:
+    """The loaded library with the signatures of the two workspace-free entry points set."""
+    global _static_ready
+    lib = load()
+    if not _static_ready:
+        P = ctypes.c_void_p
+        lib.pr2_moe_forward_static.argtypes = [ctypes.POINTER(Dims), P, P, P, P, P, P, P, P, P, P,
+                                               P, P, P, P]
+        lib.pr2_moe_forward_static.restype = ctypes.c_int
+        lib.pr2_static_scratch_bytes.argtypes = []
+        lib.pr2_static_scratch_bytes.restype = ctypes.c_size_t
+        _static_ready = True
+    return lib
+
+
+def pr2_static_scratch_bytes() -> int:
+    return int(_static_lib().pr2_static_scratch_bytes())
+
+
+def pr2_moe_forward_static(dm: Dims, h, idx, gates, W_gate, W_up, W_down, Ws_gate, Ws_up,
+                           Ws_down, out, counts=None, perm=None, status=None, stream=None) -> int:
+    """``pr2_moe_forward`` with the library's own fixed scratch array instead of a workspace:
+    for callers that cannot allocate device memory.  Calls that overlap on the GPU race."""
+    return _static_lib().pr2_moe_forward_static(
+        ctypes.byref(dm), _p(h), _p(idx), _p(gates), _p(W_gate), _p(W_up), _p(W_down),
+        _p(Ws_gate), _p(Ws_up), _p(Ws_down), _p(out), _p(counts), _p(perm), _p(status),
+        _s(stream))
