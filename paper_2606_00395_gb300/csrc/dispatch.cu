@@ -54,57 +54,108 @@ __global__ void __launch_bounds__(kDispatchChunk)
 // Exclusive block-wide scan of one int per thread (blockDim.x == 1024).
 __device__ __forceinline__ int block_exclusive_scan(int v, int* sh, int* total) {
   const int tid = threadIdx.x;
-  sh[tid] = v;
-  __syncthreads();
-  for (int o = 1; o < 1024; o <<= 1) {
-    const int add = tid >= o ? sh[tid - o] : 0;
-    __syncthreads();
-    sh[tid] += add;
-    __syncthreads();
+  const int lane = tid & 31, w = tid >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
   }
-  const int incl = sh[tid];
-  *total = sh[1023];
+  if (lane == 31) sh[w] = x;
+  __syncthreads();
+  if (w == 0) {
+    int s = sh[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, s, o);
+      if (lane >= o) s += y;
+    }
+    sh[lane] = s;  // inclusive warp totals
+  }
+  __syncthreads();
+  const int incl = x + (w > 0 ? sh[w - 1] : 0);
+  *total = sh[31];
   __syncthreads();
   return incl - v;
 }
 
+// One block of 1024 threads = G groups of N_pad threads: thread (g, e) owns expert e over the
+// block range of group g, so the per-expert scans over blocks run G-way parallel.
 __global__ void __launch_bounds__(1024)
     scan_kernel(int32_t* __restrict__ blk_hist, int nblk, int N, int64_t T, int n_shared,
                 int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
                 TileEntry* __restrict__ tiles, int32_t* __restrict__ num_tiles,
                 TileEntry* __restrict__ stiles1, TileEntry* __restrict__ stiles2) {
-  __shared__ int sh[1024];
-  const int e = threadIdx.x;
-  int total = 0;
+  __shared__ int sh[32];
+  __shared__ int part[1024];  // [G][N_pad] partial sums, then their exclusive scan over g
+  __shared__ int ex_off[kMaxExpertsDispatch + 1];
+  __shared__ int ex_tile[kMaxExpertsDispatch + 1];
+  const int tid = threadIdx.x;
+  int n_pad = 32;
+  while (n_pad < N) n_pad <<= 1;
+  const int G = 1024 / n_pad;
+  const int g = tid / n_pad, e = tid - g * n_pad;
+  const int per = (nblk + G - 1) / G;
+  const int b0 = g * per, b1 = min(nblk, b0 + per);
+  int sum = 0;
   if (e < N) {
-    for (int b = 0; b < nblk; ++b) {
-      int32_t* p = blk_hist + static_cast<int64_t>(b) * N + e;
-      const int v = *p;
-      *p = total;
+#pragma unroll 4
+    for (int b = b0; b < b1; ++b) sum += blk_hist[static_cast<int64_t>(b) * N + e];
+  }
+  part[tid] = sum;
+  __syncthreads();
+  int total = 0;
+  if (tid < N) {  // exclusive scan over the groups of expert tid
+    for (int gg = 0; gg < G; ++gg) {
+      const int v = part[gg * n_pad + tid];
+      part[gg * n_pad + tid] = total;
       total += v;
     }
-    counts[e] = total;
+    counts[tid] = total;
   }
+  __syncthreads();
   int all_rows, all_tiles;
-  const int off = block_exclusive_scan(e < N ? total : 0, sh, &all_rows);
-  const int ntile_e = e < N ? (total + kTileM - 1) / kTileM : 0;
+  const int off = block_exclusive_scan(tid < N ? total : 0, sh, &all_rows);
+  const int ntile_e = tid < N ? (total + kTileM - 1) / kTileM : 0;
   const int tstart = block_exclusive_scan(ntile_e, sh, &all_tiles);
-  if (e < N) {
-    offsets[e] = off;
-    for (int b = 0; b < nblk; ++b) blk_hist[static_cast<int64_t>(b) * N + e] += off;
-    for (int j = 0; j < ntile_e; ++j) {
-      const int r0 = off + j * kTileM;
-      const int rows = (total - j * kTileM) < kTileM ? (total - j * kTileM) : kTileM;
-      tiles[tstart + j] = TileEntry{e, r0, rows, r0};
-    }
+  if (tid < N) {
+    offsets[tid] = off;
+    ex_off[tid] = off;
+    ex_tile[tid] = tstart;
   }
-  if (e == 0) {
+  if (tid == 0) {
     offsets[N] = all_rows;
     num_tiles[0] = all_tiles;
+    ex_off[N] = all_rows;
+    ex_tile[N] = all_tiles;
+  }
+  __syncthreads();
+  // per-block bases: expert offset + rows of this expert in all earlier blocks
+  if (e < N) {
+    int run = ex_off[e] + part[g * n_pad + e];
+#pragma unroll 4
+    for (int b = b0; b < b1; ++b) {
+      int32_t* p = blk_hist + static_cast<int64_t>(b) * N + e;
+      const int v = *p;
+      *p = run;
+      run += v;
+    }
+  }
+  // M-tile table: entry i belongs to the expert whose tile range contains i
+  for (int i = tid; i < all_tiles; i += blockDim.x) {
+    int lo = 0, hi = N - 1;
+    while (lo < hi) {  // last expert with ex_tile[ex] <= i
+      const int mid = (lo + hi + 1) >> 1;
+      if (ex_tile[mid] <= i) lo = mid; else hi = mid - 1;
+    }
+    const int j = i - ex_tile[lo];
+    const int r0 = ex_off[lo] + j * kTileM;
+    const int left = ex_off[lo + 1] - r0;
+    tiles[i] = TileEntry{lo, r0, left < kTileM ? left : kTileM, r0};
   }
   // Shared experts: every token, fixed tiles.  Gate/up reads h rows, down reads Hs rows.
   const int mt_T = static_cast<int>((T + kTileM - 1) / kTileM);
-  for (int i = e; i < n_shared * mt_T; i += blockDim.x) {
+  for (int i = tid; i < n_shared * mt_T; i += blockDim.x) {
     const int j = i / mt_T, m = i - j * mt_T;
     const int r0 = m * kTileM;
     const int rows = (T - r0) < kTileM ? static_cast<int>(T - r0) : kTileM;
@@ -112,7 +163,7 @@ __global__ void __launch_bounds__(1024)
     stiles1[i] = TileEntry{j, r0, rows, o0};
     stiles2[i] = TileEntry{j, o0, rows, o0};
   }
-  if (e == 0) num_tiles[1] = n_shared * mt_T;
+  if (tid == 0) num_tiles[1] = n_shared * mt_T;
 }
 
 __global__ void __launch_bounds__(kDispatchChunk)
@@ -168,7 +219,7 @@ __global__ void __launch_bounds__(256)
   }
 }
 
-template <typename T, int V>  // V elements per 16-byte vector
+template <typename T, int V, int KMAX>  // V elements per 16-byte vector, k <= KMAX
 __global__ void __launch_bounds__(256)
     combine_kernel(const T* __restrict__ Y, const T* __restrict__ Ys,
                    const int32_t* __restrict__ inv, const float* __restrict__ gates, int64_t Tn,
@@ -184,27 +235,34 @@ __global__ void __launch_bounds__(256)
       my_pos = inv[t * k + lane];
       my_g = gates[t * k + lane];
     }
-    // The loop bound is warp-uniform so the shuffles below always see all 32 lanes.
-    for (int c0 = 0; c0 < nvec; c0 += 32) {
-      const int c = c0 + lane;
-      const bool act = c < nvec;
+    int pos[KMAX];
+    float gs[KMAX];
+#pragma unroll
+    for (int s = 0; s < KMAX; ++s) {
+      pos[s] = __shfl_sync(0xffffffffu, my_pos, s);
+      gs[s] = __shfl_sync(0xffffffffu, my_g, s);
+      if (s >= k) pos[s] = -1;
+    }
+    for (int c = lane; c < nvec; c += 32) {
+      uint4 raw[KMAX];
+#pragma unroll
+      for (int s = 0; s < KMAX; ++s)
+        if (pos[s] >= 0)
+          raw[s] = __ldg(reinterpret_cast<const uint4*>(Y + static_cast<int64_t>(pos[s]) * d) + c);
       float acc[V];
 #pragma unroll
       for (int j = 0; j < V; ++j) acc[j] = 0.f;
-      for (int s = 0; s < k; ++s) {
-        const int p = __shfl_sync(0xffffffffu, my_pos, s);
-        const float gs = __shfl_sync(0xffffffffu, my_g, s);
-        if (p < 0 || !act) continue;
-        const uint4 raw = __ldg(reinterpret_cast<const uint4*>(Y + static_cast<int64_t>(p) * d) + c);
-        const T* v = reinterpret_cast<const T*>(&raw);
 #pragma unroll
-        for (int j = 0; j < V; ++j) acc[j] = fmaf(gs, to_f32<T>(v[j]), acc[j]);
+      for (int s = 0; s < KMAX; ++s) {
+        if (pos[s] < 0) continue;
+        const T* v = reinterpret_cast<const T*>(&raw[s]);
+#pragma unroll
+        for (int j = 0; j < V; ++j) acc[j] = fmaf(gs[s], to_f32<T>(v[j]), acc[j]);
       }
-      if (!act) continue;
       for (int j2 = 0; j2 < n_shared; ++j2) {
-        const uint4 raw = __ldg(
+        const uint4 r = __ldg(
             reinterpret_cast<const uint4*>(Ys + (static_cast<int64_t>(j2) * Tn + t) * d) + c);
-        const T* v = reinterpret_cast<const T*>(&raw);
+        const T* v = reinterpret_cast<const T*>(&r);
 #pragma unroll
         for (int j = 0; j < V; ++j) acc[j] += to_f32<T>(v[j]);
       }
@@ -247,12 +305,20 @@ cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st) {
   int64_t blocks = (a.T + 7) / 8;
   const int64_t cap = static_cast<int64_t>(num_sms) * 8;
   if (blocks > cap) blocks = cap;
-  if (a.bf16) {
-    combine_kernel<__nv_bfloat16, 8><<<static_cast<int>(blocks), 256, 0, st>>>(
+  if (a.bf16 && a.k <= 8) {
+    combine_kernel<__nv_bfloat16, 8, 8><<<static_cast<int>(blocks), 256, 0, st>>>(
         static_cast<const __nv_bfloat16*>(a.Y), static_cast<const __nv_bfloat16*>(a.Ys), a.inv,
         a.gates, a.T, a.k, a.d, a.n_shared, static_cast<__nv_bfloat16*>(a.out));
+  } else if (a.bf16) {
+    combine_kernel<__nv_bfloat16, 8, 32><<<static_cast<int>(blocks), 256, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(a.Y), static_cast<const __nv_bfloat16*>(a.Ys), a.inv,
+        a.gates, a.T, a.k, a.d, a.n_shared, static_cast<__nv_bfloat16*>(a.out));
+  } else if (a.k <= 8) {
+    combine_kernel<float, 4, 8><<<static_cast<int>(blocks), 256, 0, st>>>(
+        static_cast<const float*>(a.Y), static_cast<const float*>(a.Ys), a.inv, a.gates, a.T,
+        a.k, a.d, a.n_shared, static_cast<float*>(a.out));
   } else {
-    combine_kernel<float, 4><<<static_cast<int>(blocks), 256, 0, st>>>(
+    combine_kernel<float, 4, 32><<<static_cast<int>(blocks), 256, 0, st>>>(
         static_cast<const float*>(a.Y), static_cast<const float*>(a.Ys), a.inv, a.gates, a.T,
         a.k, a.d, a.n_shared, static_cast<float*>(a.out));
   }

@@ -5,7 +5,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include "../../include/pr2.h"
+#include "pr2.h"
 
 namespace pr2 {
 
