@@ -38,8 +38,8 @@ FLUSH_BYTES = 512 << 20
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["pr2", "reference"], default="pr2")
     ap.add_argument("--workload", default="qwen3_30b_a3b", choices=sorted(synth.CONFIGS))
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -56,6 +56,23 @@ def peaks():
                     bf16_sustained=float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
                     source="measured")
     return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
+
+
+def measured_traffic(kernel_key: str):
+    """DRAM bytes per launch of a kernel from the committed ncu summary, or None when any source
+    file the capture was taken with has changed since (the counters no longer apply)."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    entry = json.load(open(path)).get(kernel_key)
+    if not entry:
+        return None
+    for rel, digest in entry["sources_sha256"].items():
+        f = os.path.join(ROOT, rel)
+        if not os.path.exists(f) or hashlib.sha256(open(f, "rb").read()).hexdigest() != digest:
+            return None
+    return entry["dram_bytes_per_launch"]
 
 
 def workload_desc(cfg):
@@ -83,7 +100,7 @@ class ClockSampler:
             self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", sel, f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.fh,
+                 "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.fh,
                 stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
@@ -290,7 +307,8 @@ def run_pr2(args, rank, world, local_rank):
     dom = max(("gate_up", "down"), key=lambda n: kernels[n]["ms"])
     dk = kernels[dom]
     roofline = dict(kernel=f"expert_tc_kernel ({dom})", bound=dk["bound"], achieved=dk["achieved"],
-                    peak=dk["peak"], unit=dk["unit"], frac=dk["frac"], traffic=None,
+                    peak=dk["peak"], unit=dk["unit"], frac=dk["frac"],
+                    traffic=measured_traffic(f"{cfg.name}/{dom}"),
                     peak_source=f"{pk['source']} (MEASURED_PEAKS.json burst)"
                     if pk["source"] == "measured" else "fallback",
                     algorithmic=("flops" if dk["bound"] == "tensor" else "bytes"),
