@@ -157,6 +157,9 @@ pr2_status route_common(const pr2_dims* dims, bool predict, const void* h, const
                             idx_out, gates, aux, near_tie, status_dev, st);
   } else {
     if (dm.T > (int64_t{1} << 30)) return PR2_ERR_UNSUPPORTED;
+    const int num_sms = num_sms_of_current_device();
+    if (num_sms <= 0) return PR2_ERR_CUDA;
+    const int split = route_split(static_cast<int>(dm.T), dm.N, dm.d, predict, num_sms);
     CUtensorMap tm_h, tm_w, tm_wp;
     if (!make_tmap_bf16(&tm_h, h, dm.d, dm.T, 64, kTileM) ||
         !make_tmap_bf16(&tm_w, W, dm.d, dm.N, 64, dm.N))
@@ -168,7 +171,7 @@ pr2_status route_common(const pr2_dims* dims, bool predict, const void* h, const
     }
     RouteTcArgs a{static_cast<int>(dm.T), dm.d, dm.N, dm.k, idx_in, idx_out,
                   gates, aux, near_tie, status_dev};
-    err = launch_route_tc(predict, tm_h, tm_w, tm_wp, a, st);
+    err = launch_route_tc(predict, tm_h, tm_w, tm_wp, a, split, st);
   }
   return finish(err, dm.flags, status_dev, st);
 }

@@ -251,6 +251,10 @@ __device__ __forceinline__ void st_cluster_v4(uint32_t addr, uint32_t a, uint32_
                "r"(c), "r"(d)
                : "memory");
 }
+__device__ __forceinline__ void st_cluster_v2(uint32_t addr, uint32_t a, uint32_t b) {
+  asm volatile("st.shared::cluster.v2.b32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b)
+               : "memory");
+}
 
 // ------------------------------------------------------------------------------------------
 // Small numeric and load/store helpers.

@@ -37,8 +37,11 @@ struct RouteTcArgs {
   int64_t* near_tie;
   int32_t* status;
 };
+// CTAs of the cluster that splits K for one 128-token tile (1 = no split).
+int route_split(int T, int N, int d, bool predict, int num_sms);
 cudaError_t launch_route_tc(bool predict, const CUtensorMap& tm_h, const CUtensorMap& tm_w,
-                            const CUtensorMap& tm_wp, const RouteTcArgs& a, cudaStream_t st);
+                            const CUtensorMap& tm_wp, const RouteTcArgs& a, int split,
+                            cudaStream_t st);
 
 // ---- dispatch and combine (dispatch.cu) ----------------------------------------------------
 struct DispatchArgs {

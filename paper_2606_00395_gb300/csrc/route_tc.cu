@@ -1,17 +1,33 @@
-// bf16 routing on the tcgen05 tensor cores.  One CTA = 128 tokens.
+// bf16 routing on the tcgen05 tensor cores.
 //
 //   predict (Eqs. pr2_predict, pr2_route; Algorithm 2 first two steps):
-//     [p_old | b] = h [W ; W_p]^T   one M=128 x N=2N accumulator in TMEM (fp32), K = d,
+//     [p_old | b] = h [W ; W_p]^T   (fp32 accumulators in TMEM, K = d),
 //     z = p_old + b, rho_hat = Softmax(z), idx = TopK(rho_hat, k), gates = rho_hat[idx],
 //     p_old optionally written as the feature-cache logits.
 //   replay (Sec. 4.1 "Replay During Training"):
 //     p = h W^T, rho = Softmax(p), gates = rho[idx_in]   (no top-k, no predictor).
 //
-// Warp roles: warp 0 = TMA producer (h tile + weight tile per 64-wide K block), warp 1 = TMEM
-// owner and MMA issuer, warps 2..5 = epilogue, one thread per token row (TMEM lane).
-// The epilogue selects on z in fp32 (softmax is monotone, so the order equals the order of
-// rho_hat); ties go to the lower expert index.
+// A 128-token tile is handled by a cluster of S CTAs (S = 1, 2, 4 or 8) that split K = d.  Each
+// tcgen05.mma costs the same issue time for any N <= 256 (one M=128 x N x K=16 step), so a lone
+// tile's chain of d/16 MMAs, not bandwidth, bounds it, and only a K split shortens that chain:
+// CTA r multiplies K blocks [r KB/S, (r+1) KB/S) into a partial [128 x NB] fp32 accumulator
+// (NB = 2N columns [p_old | b] for predict, N for replay).
+//
+// Warp roles: warp 0 = TMA producer, warp 1 = TMEM owner and MMA issuer, warps 2..5 = epilogue.
+// With S > 1 the partials are reduce-scattered by rows through distributed shared memory: CTA q
+// receives rows [q 128/S, (q+1) 128/S) of every CTA's partial, stored [source][column/4][row][4]
+// so that each warp store moves contiguous bytes, and sums them in source order (deterministic).
+// Each row is then finished by S consecutive threads, thread `part` owning experts
+// [part N/S, (part+1) N/S); with S = 1 one thread finishes its row straight from TMEM.  A thread
+// reduces its experts to a max, a sum of exp(z - max) and (predict) its top-16 by 64-bit keys
+// (orderable z bits, inverted expert index: z descending, ties to the lower expert), built by
+// bitonic sorting 16 experts at a time and merging, in one pass with a running (online) softmax
+// sum; the S threads of a row then combine max and sum (sum_q s_q exp(m_q - max), fixed shuffle
+// order) and merge their lists by shuffles.
+// Selection is on z in fp32 (softmax is monotone, so the order equals the order of rho_hat).
 #include <float.h>
+
+#include <mutex>
 
 #include "pr2_device.cuh"
 #include "pr2_internal.h"
@@ -23,6 +39,8 @@ constexpr int kThreads = 192;
 constexpr int kBK = 64;                          // bf16 elements per 128-byte swizzle row
 constexpr int kATileBytes = kTileM * kBK * 2;    // 16 KB
 constexpr int kKeep = kMaxTopK + 1;              // top-(k+1) kept for the margin
+constexpr int kMaxSplit = 8;
+constexpr int kMaxStages = 12;
 
 struct RouteSmemLayout {
   int stages;
@@ -36,13 +54,17 @@ __host__ __device__ inline RouteSmemLayout route_layout(int N, bool predict) {
   RouteSmemLayout L;
   L.b_rows = predict ? 2 * N : N;
   L.stage_bytes = kATileBytes + L.b_rows * kBK * 2;
-  L.stages = (200 * 1024) / L.stage_bytes;
-  if (L.stages > 6) L.stages = 6;
+  L.stages = (192 * 1024) / L.stage_bytes;
+  if (L.stages > kMaxStages) L.stages = kMaxStages;
   if (L.stages < 2) L.stages = 2;
   L.bar_offset = L.stages * L.stage_bytes;
   L.total = 1024 + L.bar_offset + 256;
   return L;
 }
+
+// Bytes of the reduce-scatter buffer, [S][NB/S/4][128][4] fp32, placed over the pipeline
+// stages once every CTA of the cluster has finished its K blocks.
+__host__ __device__ inline int route_recv_bytes(int b_rows) { return b_rows * kTileM * 4; }
 
 __host__ __device__ inline uint32_t tmem_cols_for(int cols) {
   uint32_t c = 32;
@@ -50,25 +72,111 @@ __host__ __device__ inline uint32_t tmem_cols_for(int cols) {
   return c;
 }
 
+// Compare-exchange leaving the larger key in a.
+__device__ __forceinline__ void cas_desc(uint64_t& a, uint64_t& b) {
+  const bool sw = b > a;
+  const uint64_t hi = sw ? b : a;
+  const uint64_t lo = sw ? a : b;
+  a = hi;
+  b = lo;
+}
+
+// Bitonic sort of 16 keys into descending order.
+__device__ __forceinline__ void sort16_desc(uint64_t (&v)[16]) {
+#pragma unroll
+  for (int kk = 2; kk <= 16; kk <<= 1)
+#pragma unroll
+    for (int j = kk >> 1; j > 0; j >>= 1)
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int l = i ^ j;
+        if (l > i) {
+          if ((i & kk) == 0)
+            cas_desc(v[i], v[l]);
+          else
+            cas_desc(v[l], v[i]);
+        }
+      }
+}
+
+// top <- the 16 largest of top and c, both sorted descending (c is clobbered): the elementwise
+// max of top and reversed c is a bitonic sequence holding them, then a bitonic merge sorts it.
+__device__ __forceinline__ void merge16_desc(uint64_t (&top)[16], const uint64_t (&c)[16]) {
+#pragma unroll
+  for (int i = 0; i < 16; ++i) top[i] = top[i] > c[15 - i] ? top[i] : c[15 - i];
+#pragma unroll
+  for (int j = 8; j > 0; j >>= 1)
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const int l = i ^ j;
+      if (l > i) cas_desc(top[i], top[l]);
+    }
+}
+
+// 64-bit key ordering (z descending, expert ascending).  An empty slot is key 0, below every
+// real key.
+__device__ __forceinline__ uint64_t topk_key(float z, int e) {
+  const uint32_t u = __float_as_uint(z);
+  const uint32_t ord = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  return (static_cast<uint64_t>(ord) << 32) | static_cast<uint32_t>(~static_cast<uint32_t>(e));
+}
+__device__ __forceinline__ float key_z(uint64_t key) {
+  const uint32_t ord = static_cast<uint32_t>(key >> 32);
+  return __uint_as_float((ord & 0x80000000u) ? (ord & 0x7fffffffu) : ~ord);
+}
+__device__ __forceinline__ int key_e(uint64_t key) {
+  return static_cast<int>(~static_cast<uint32_t>(key));
+}
+
+// Write a finished predict row: idx and gates of the k best keys; returns the near-tie flag
+// rho_hat_(k) - rho_hat_(k+1) < PR2_NEAR_TIE_GAP.
+__device__ __forceinline__ bool predict_write(const uint64_t (&key)[16], float mx, float inv_s,
+                                              int64_t t, const RouteTcArgs& a) {
+  int32_t* irow = a.idx_out + t * a.k;
+  float* grow = a.gates + t * a.k;
+  float pk = 0.f, pk1 = 0.f;
+#pragma unroll
+  for (int j = 0; j < kKeep; ++j) {
+    const float pr = expf(key_z(key[j]) - mx) * inv_s;
+    if (j < a.k) {
+      irow[j] = key_e(key[j]);
+      grow[j] = pr;
+    }
+    if (j == a.k - 1) pk = pr;
+    if (j == a.k) pk1 = pr;
+  }
+  return (a.k < a.N) && (pk - pk1 < (float)PR2_NEAR_TIE_GAP);
+}
+
+template <bool predict, int split>
 __global__ void __launch_bounds__(kThreads, 1)
     route_tc_kernel(const __grid_constant__ CUtensorMap tm_h,
                     const __grid_constant__ CUtensorMap tm_w,
-                    const __grid_constant__ CUtensorMap tm_wp, RouteTcArgs a, int predict) {
-  extern __shared__ uint8_t smem_raw[];
-  const RouteSmemLayout L = route_layout(a.N, predict != 0);
-  uint8_t* smem = reinterpret_cast<uint8_t*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+                    const __grid_constant__ CUtensorMap tm_wp, RouteTcArgs a) {
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  const int N = a.N, k = a.k;
+  const RouteSmemLayout L = route_layout(N, predict);
+  // 1024-B aligned base, kept as an offset into the shared array so the compiler knows every
+  // derived pointer is shared memory.
+  const uint32_t pad = (1024u - (smem_u32(smem_raw) & 1023u)) & 1023u;
+  uint8_t* smem = smem_raw + pad;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bar_offset);
   uint64_t* empty = full + L.stages;
   uint64_t* acc_full = empty + L.stages;
   uint64_t* drain = acc_full + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const float4* recv = reinterpret_cast<const float4*>(smem);  // valid after the exchange
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int t0 = blockIdx.x * kTileM;
-  const int KB = a.d / kBK;
+  const int rank = split > 1 ? static_cast<int>(cluster_ctarank()) : 0;
+  const int t0 = (blockIdx.x / split) * kTileM;
+  const int R = kTileM / split;             // rows finished by this CTA
+  const int nr = N / split;                 // experts of one finishing thread
+  const int nb4 = L.b_rows / 4;             // float4 columns of a partial row
+  const int KBper = (a.d / kBK) / split;
+  const int kb0 = rank * KBper, kb1 = kb0 + KBper;
   const uint32_t ncols = tmem_cols_for(L.b_rows);
 
   if (threadIdx.x == 0) {
@@ -92,91 +200,189 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 0 && lane == 0) {
-    // ---------------- TMA producer ----------------
-    const uint32_t bytes = static_cast<uint32_t>(L.stage_bytes);
-    uint32_t issued = 0, last_par = 0;
-    int stage = 0;
-    uint32_t phase = 0;
-    const uint64_t keep = l2_policy_evict_last();    // weights are re-read by every CTA
-    const uint64_t stream = l2_policy_evict_first(); // h is read once
-    for (int kb = 0; kb < KB; ++kb) {
-      if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, a.status)) break;
-      uint8_t* sa = smem + stage * L.stage_bytes;
-      uint8_t* sb = sa + kATileBytes;
-      mbar_arrive_expect_tx(&full[stage], bytes);
-      tma_load_2d_hint(sa, &tm_h, &full[stage], kb * kBK, t0, stream);
-      tma_load_2d_hint(sb, &tm_w, &full[stage], kb * kBK, 0, keep);
-      if (predict) tma_load_2d_hint(sb + a.N * kBK * 2, &tm_wp, &full[stage], kb * kBK, 0, keep);
-      issued |= 1u << stage;
-      last_par = (last_par & ~(1u << stage)) | (phase << stage);
-      if (++stage == L.stages) {
-        stage = 0;
-        phase ^= 1u;
-      }
-    }
-    // Drain: every issued copy must have landed before the CTA can exit.
-    for (int s = 0; s < L.stages; ++s)
-      if ((issued >> s) & 1u)
-        mbar_wait_slow(&full[s], (last_par >> s) & 1u, nullptr, nullptr, kDrainLimitNs);
-  } else if (warp == 1 && lane == 0) {
-    // ---------------- MMA issuer ----------------
-    int stage = 0;
-    uint32_t phase = 0;
-    bool ok = true;
-    for (int kb = 0; kb < KB && ok; ++kb) {
-      if (!mbar_wait(&full[stage], phase, abort_flag, a.status)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      const uint32_t sa = smem_u32(smem + stage * L.stage_bytes);
-      const uint32_t sb = sa + kATileBytes;
-#pragma unroll
-      for (int kk = 0; kk < kBK / 16; ++kk) {
-        const uint64_t adesc = umma_desc_sw128(sa + kk * 32);
-        for (int n0 = 0; n0 < L.b_rows; n0 += 256) {
-          const int nc = (L.b_rows - n0) < 256 ? (L.b_rows - n0) : 256;
-          const uint64_t bdesc = umma_desc_sw128(sb + n0 * (kBK * 2) + kk * 32);
-          umma_bf16(tmem + n0, adesc, bdesc, umma_idesc_bf16(kTileM, nc),
-                    (kb > 0 || kk > 0) ? 1u : 0u);
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      const uint32_t bytes = static_cast<uint32_t>(L.stage_bytes);
+      uint32_t issued = 0, last_par = 0;
+      int stage = 0;
+      uint32_t phase = 0;
+      const uint64_t keep = l2_policy_evict_last();    // weights are re-read by every tile
+      const uint64_t once = l2_policy_evict_first();   // h is read once
+      for (int kb = kb0; kb < kb1; ++kb) {
+        if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, a.status)) break;
+        uint8_t* sa = smem + stage * L.stage_bytes;
+        uint8_t* sb = sa + kATileBytes;
+        mbar_arrive_expect_tx(&full[stage], bytes);
+        tma_load_2d_hint(sa, &tm_h, &full[stage], kb * kBK, t0, once);
+        tma_load_2d_hint(sb, &tm_w, &full[stage], kb * kBK, 0, keep);
+        if (predict) tma_load_2d_hint(sb + N * kBK * 2, &tm_wp, &full[stage], kb * kBK, 0, keep);
+        issued |= 1u << stage;
+        last_par = (last_par & ~(1u << stage)) | (phase << stage);
+        if (++stage == L.stages) {
+          stage = 0;
+          phase ^= 1u;
         }
       }
-      umma_commit(&empty[stage]);
-      if (++stage == L.stages) {
-        stage = 0;
-        phase ^= 1u;
+      // Drain: every issued copy must have landed before the stages are reused or the CTA exits.
+      for (int s = 0; s < L.stages; ++s)
+        if ((issued >> s) & 1u)
+          mbar_wait_slow(&full[s], (last_par >> s) & 1u, nullptr, nullptr, kDrainLimitNs);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int kb = kb0; kb < kb1 && ok; ++kb) {
+        if (!mbar_wait(&full[stage], phase, abort_flag, a.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t sa = smem_u32(smem + stage * L.stage_bytes);
+        const uint32_t sb = sa + kATileBytes;
+#pragma unroll
+        for (int kk = 0; kk < kBK / 16; ++kk) {
+          const uint64_t adesc = umma_desc_sw128(sa + kk * 32);
+          for (int n0 = 0; n0 < L.b_rows; n0 += 256) {
+            const int nc = (L.b_rows - n0) < 256 ? (L.b_rows - n0) : 256;
+            const uint64_t bdesc = umma_desc_sw128(sb + n0 * (kBK * 2) + kk * 32);
+            umma_bf16(tmem + n0, adesc, bdesc, umma_idesc_bf16(kTileM, nc),
+                      (kb > kb0 || kk > 0) ? 1u : 0u);
+          }
+        }
+        umma_commit(&empty[stage]);
+        if (++stage == L.stages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (ok) umma_commit(acc_full);
+      umma_commit(drain);
+      mbar_wait_slow(drain, 0, nullptr, nullptr, kDrainLimitNs);
+    }
+    __syncwarp();
+  }
+
+  // ---------------- epilogue ----------------
+  const bool epi = warp >= 2;
+  const int q = warp & 3;
+  const int row = q * 32 + lane;  // TMEM lane of this thread
+  const uint32_t trow = tmem + (static_cast<uint32_t>(q * 32) << 16);
+  // Finishing coordinates: row lr of this CTA's R rows, experts [part nr, (part+1) nr).
+  const int et = threadIdx.x - 64;
+  const int lr = split == 1 ? row : et / split;
+  const int part = split == 1 ? 0 : et - lr * split;
+  const int fe0 = part * nr;
+  const int64_t t = static_cast<int64_t>(t0) + static_cast<int64_t>(rank) * R + lr;
+  const bool live = epi && t < a.T;
+
+  // replay: cached indices, validated (range, duplicates) while the K blocks run
+  int e_s[kMaxTopK];
+  bool bad = false;
+  if (!predict) {
+#pragma unroll
+    for (int s = 0; s < kMaxTopK; ++s) {
+      int e = -1;
+      if (live && s < k) {
+        e = a.idx_in[t * k + s];
+        bool ok = e >= 0 && e < N;
+#pragma unroll
+        for (int s2 = 0; s2 < kMaxTopK; ++s2)
+          if (s2 < s && e_s[s2] == e) ok = false;
+        if (!ok) {
+          bad = true;
+          e = -1;
+        }
+      }
+      e_s[s] = e;
+    }
+  }
+
+  bool have = false;
+  if (epi) {
+    // tcgen05.ld is warp-collective: the whole warp reads TMEM or none of it does.
+    have = __all_sync(0xffffffffu, mbar_wait(acc_full, 0, abort_flag, a.status));
+    if (have) tc_fence_after();
+  }
+  if (split > 1) {
+    cluster_sync();  // every CTA has finished its K blocks: the pipeline stages are free
+    if (epi && have) {
+      // Reduce-scatter by rows: this TMEM row goes to CTA row / R as its row row % R.
+      float4* recv_w = reinterpret_cast<float4*>(smem);
+      const uint32_t dst = static_cast<uint32_t>(row / R);
+      const int drow = row - static_cast<int>(dst) * R;
+      const uint32_t rbase =
+          mapa_shared(smem_u32(recv_w + (rank * nb4) * R + drow), dst);
+      for (int c0 = 0; c0 < L.b_rows; c0 += 32) {
+        uint32_t r0[16], r1[16];
+        tmem_ld16(trow + c0, r0);
+        tmem_ld16(trow + c0 + 16, r1);
+        tmem_wait_ld(r0);
+        reg_fence(r1);
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          st_cluster_v4(rbase + static_cast<uint32_t>(((c0 / 4 + j) * R) * 16), r0[4 * j],
+                        r0[4 * j + 1], r0[4 * j + 2], r0[4 * j + 3]);
+        if (c0 + 16 < L.b_rows) {  // b_rows is a multiple of 16, not always of 32
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            st_cluster_v4(rbase + static_cast<uint32_t>(((c0 / 4 + 4 + j) * R) * 16), r1[4 * j],
+                          r1[4 * j + 1], r1[4 * j + 2], r1[4 * j + 3]);
+        }
       }
     }
-    if (ok) umma_commit(acc_full);
-    umma_commit(drain);
-    mbar_wait_slow(drain, 0, nullptr, nullptr, kDrainLimitNs);
-  } else if (warp >= 2) {
-    // ---------------- epilogue: one thread per token ----------------
-    const int q = warp & 3;
-    const int row = q * 32 + lane;
-    const int t = t0 + row;
-    const bool live = t < a.T;
-    const uint32_t trow = tmem + (static_cast<uint32_t>(q * 32) << 16);
-    if (mbar_wait(acc_full, 0, abort_flag, a.status)) {
-      tc_fence_after();
-      const int N = a.N, k = a.k;
-      if (predict) {
-        float tv[kKeep];
-        int ti[kKeep];
+    cluster_sync();  // every partial row has landed
+  }
+  // Columns [c, c + 16) of the finished row: summed partials (S > 1) or TMEM (S = 1).
+  auto load16 = [&](int c, uint32_t (&r)[16]) {
+    if (split == 1) {
+      tmem_ld16(trow + c, r);
+      tmem_wait_ld(r);
+      return;
+    }
 #pragma unroll
-        for (int j = 0; j < kKeep; ++j) {
-          tv[j] = -FLT_MAX;
-          ti[j] = 0x7fffffff;
-        }
-        float* lrow = a.logits_or_probs ? a.logits_or_probs + static_cast<int64_t>(t) * N : nullptr;
-        for (int c0 = 0; c0 < N; c0 += 16) {
+    for (int j = 0; j < 4; ++j) {
+      float4 v = recv[(c / 4 + j) * R + lr];
+#pragma unroll
+      for (int src = 1; src < split; ++src) {
+        const float4 w = recv[(src * nb4 + c / 4 + j) * R + lr];
+        v.x += w.x;
+        v.y += w.y;
+        v.z += w.z;
+        v.w += w.w;
+      }
+      r[4 * j] = __float_as_uint(v.x);
+      r[4 * j + 1] = __float_as_uint(v.y);
+      r[4 * j + 2] = __float_as_uint(v.z);
+      r[4 * j + 3] = __float_as_uint(v.w);
+    }
+  };
+
+  // One pass over this thread's experts, 16 at a time: running max m and sum of exp(z - m),
+  // (predict) the top-16 keys, (replay) the z of the cached slots.
+  if (epi) {
+    bool tie = false;
+    float m = -FLT_MAX, sum = 0.f;
+    uint64_t top[16];
+    float z_s[kMaxTopK];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) top[j] = 0ull;
+#pragma unroll
+    for (int s = 0; s < kMaxTopK; ++s) z_s[s] = 0.f;
+    if (have) {
+      float* lrow = (predict && a.logits_or_probs != nullptr && live) ? a.logits_or_probs + t * N
+                                                                      : nullptr;
+      for (int c0 = fe0; c0 < fe0 + nr; c0 += 16) {
+        float z[16];
+        if (predict) {
           uint32_t rp[16], rb[16];
-          tmem_ld16(trow + c0, rp);
-          tmem_ld16(trow + N + c0, rb);
-          tmem_wait_ld(rp);
-          reg_fence(rb);
-          if (live && lrow != nullptr) {
+          load16(c0, rp);
+          load16(N + c0, rb);
+          if (lrow != nullptr) {
             float4* dst = reinterpret_cast<float4*>(lrow + c0);
 #pragma unroll
             for (int j = 0; j < 4; ++j)
@@ -184,128 +390,88 @@ __global__ void __launch_bounds__(kThreads, 1)
                                    __uint_as_float(rp[4 * j + 2]), __uint_as_float(rp[4 * j + 3]));
           }
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            float cv = __uint_as_float(rp[j]) + __uint_as_float(rb[j]);
-            if (cv > tv[kKeep - 1]) {
-              int ci = c0 + j;
-#pragma unroll
-              for (int s = 0; s < kKeep; ++s) {
-                const bool sw = cv > tv[s];
-                const float ov = tv[s];
-                const int oi = ti[s];
-                tv[s] = sw ? cv : ov;
-                ti[s] = sw ? ci : oi;
-                cv = sw ? ov : cv;
-                ci = sw ? oi : ci;
-              }
-            }
-          }
-        }
-        const float mx = tv[0];
-        float sum = 0.f;
-        for (int c0 = 0; c0 < N; c0 += 16) {
-          uint32_t rp[16], rb[16];
-          tmem_ld16(trow + c0, rp);
-          tmem_ld16(trow + N + c0, rb);
-          tmem_wait_ld(rp);
-          reg_fence(rb);
-#pragma unroll
-          for (int j = 0; j < 16; ++j)
-            sum += expf(__uint_as_float(rp[j]) + __uint_as_float(rb[j]) - mx);
-        }
-        const float inv_s = 1.0f / sum;
-        bool tie = false;
-        if (live) {
-          int32_t* irow = a.idx_out + static_cast<int64_t>(t) * k;
-          float* grow = a.gates + static_cast<int64_t>(t) * k;
-          float pk = 0.f, pk1 = 0.f;
-#pragma unroll
-          for (int s = 0; s < kKeep; ++s) {
-            const float pr = expf(tv[s] - mx) * inv_s;
-            if (s < k) {
-              irow[s] = ti[s];
-              grow[s] = pr;
-            }
-            if (s == k - 1) pk = pr;
-            if (s == k) pk1 = pr;
-          }
-          tie = (k < N) && (pk - pk1 < (float)PR2_NEAR_TIE_GAP);
-        }
-        const unsigned ties = __ballot_sync(0xffffffffu, tie);
-        if (lane == 0 && ties != 0u && a.near_tie != nullptr)
-          atomicAdd(reinterpret_cast<unsigned long long*>(a.near_tie),
-                    static_cast<unsigned long long>(__popc(ties)));
-      } else {
-        // replay: cached indices, validated, their probabilities captured in the second pass
-        int e_s[kMaxTopK];
-        float z_s[kMaxTopK];
-        bool bad = false;
-#pragma unroll
-        for (int s = 0; s < kMaxTopK; ++s) {
-          int e = -1;
-          if (live && s < k) {
-            e = a.idx_in[static_cast<int64_t>(t) * k + s];
-            bool ok = e >= 0 && e < N;
-#pragma unroll
-            for (int s2 = 0; s2 < kMaxTopK; ++s2)
-              if (s2 < s && e_s[s2] == e) ok = false;
-            if (!ok) {
-              bad = true;
-              e = -1;
-            }
-          }
-          e_s[s] = e;
-          z_s[s] = 0.f;
-        }
-        float mx = -FLT_MAX;
-        for (int c0 = 0; c0 < N; c0 += 16) {
+          for (int j = 0; j < 16; ++j) z[j] = __uint_as_float(rp[j]) + __uint_as_float(rb[j]);
+        } else {
           uint32_t rp[16];
-          tmem_ld16(trow + c0, rp);
-          tmem_wait_ld(rp);
-#pragma unroll
-          for (int j = 0; j < 16; ++j) mx = fmaxf(mx, __uint_as_float(rp[j]));
-        }
-        float sum = 0.f;
-        for (int c0 = 0; c0 < N; c0 += 16) {
-          uint32_t rp[16];
-          tmem_ld16(trow + c0, rp);
-          tmem_wait_ld(rp);
+          load16(c0, rp);
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
-            const float z = __uint_as_float(rp[j]);
-            sum += expf(z - mx);
+            z[j] = __uint_as_float(rp[j]);
 #pragma unroll
             for (int s = 0; s < kMaxTopK; ++s)
-              if (e_s[s] == c0 + j) z_s[s] = z;
+              if (e_s[s] == c0 + j) z_s[s] = z[j];
           }
         }
-        const float inv_s = 1.0f / sum;
-        if (live) {
-          float* grow = a.gates + static_cast<int64_t>(t) * k;
+        float cm = z[0];
 #pragma unroll
-          for (int s = 0; s < kMaxTopK; ++s)
-            if (s < k) grow[s] = (e_s[s] >= 0) ? expf(z_s[s] - mx) * inv_s : 0.f;
-          if (bad && a.status != nullptr) atomicOr(a.status, PR2_STATUS_BAD_INDEX);
+        for (int j = 1; j < 16; ++j) cm = fmaxf(cm, z[j]);
+        const float nm = fmaxf(m, cm);
+        float cs = 0.f;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) cs += expf(z[j] - nm);
+        sum = sum * expf(m - nm) + cs;
+        m = nm;
+        if (predict) {
+          uint64_t ck[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) ck[j] = topk_key(z[j], c0 + j);
+          sort16_desc(ck);
+          merge16_desc(top, ck);
         }
-        if (a.logits_or_probs != nullptr) {
-          float* prow = a.logits_or_probs + static_cast<int64_t>(t) * N;
-          for (int c0 = 0; c0 < N; c0 += 16) {
-            uint32_t rp[16];
-            tmem_ld16(trow + c0, rp);
-            tmem_wait_ld(rp);
-            if (live) {
-              float4* dst = reinterpret_cast<float4*>(prow + c0);
+      }
+    }
+    // Combine the S threads of the row (consecutive lanes): max, rescaled sum, merged lists.
+    float mx = m;
 #pragma unroll
-              for (int j = 0; j < 4; ++j)
-                dst[j] = make_float4(expf(__uint_as_float(rp[4 * j]) - mx) * inv_s,
-                                     expf(__uint_as_float(rp[4 * j + 1]) - mx) * inv_s,
-                                     expf(__uint_as_float(rp[4 * j + 2]) - mx) * inv_s,
-                                     expf(__uint_as_float(rp[4 * j + 3]) - mx) * inv_s);
-            }
+    for (int o = 1; o < split; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    float fs = have ? sum * expf(m - mx) : 0.f;
+#pragma unroll
+    for (int o = 1; o < split; o <<= 1) fs += __shfl_xor_sync(0xffffffffu, fs, o);
+    const float inv_s = 1.0f / fs;
+    if (predict) {
+#pragma unroll
+      for (int o = 1; o < split; o <<= 1) {
+        uint64_t other[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          other[j] = j < kKeep ? __shfl_xor_sync(0xffffffffu, top[j], o) : 0ull;
+        merge16_desc(top, other);
+      }
+      if (have && live && part == 0) tie = predict_write(top, mx, inv_s, t, a);
+    } else {
+      // Each valid slot's z is held by the one thread owning its expert; the others hold 0.
+#pragma unroll
+      for (int s = 0; s < kMaxTopK; ++s)
+#pragma unroll
+        for (int o = 1; o < split; o <<= 1) z_s[s] += __shfl_xor_sync(0xffffffffu, z_s[s], o);
+      if (have && live && part == 0) {
+        float* grow = a.gates + t * k;
+#pragma unroll
+        for (int s = 0; s < kMaxTopK; ++s)
+          if (s < k) grow[s] = (e_s[s] >= 0) ? expf(z_s[s] - mx) * inv_s : 0.f;
+        if (bad && a.status != nullptr) atomicOr(a.status, PR2_STATUS_BAD_INDEX);
+      }
+      if (have && a.logits_or_probs != nullptr) {
+        float* prow = a.logits_or_probs + t * N;
+        for (int c0 = fe0; c0 < fe0 + nr; c0 += 16) {
+          uint32_t rp[16];
+          load16(c0, rp);
+          if (live) {
+            float4* dst = reinterpret_cast<float4*>(prow + c0);
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              dst[j] = make_float4(expf(__uint_as_float(rp[4 * j]) - mx) * inv_s,
+                                   expf(__uint_as_float(rp[4 * j + 1]) - mx) * inv_s,
+                                   expf(__uint_as_float(rp[4 * j + 2]) - mx) * inv_s,
+                                   expf(__uint_as_float(rp[4 * j + 3]) - mx) * inv_s);
           }
         }
       }
     }
+    const unsigned ties = __ballot_sync(0xffffffffu, tie);
+    if (lane == 0 && ties != 0u && a.near_tie != nullptr)
+      atomicAdd(reinterpret_cast<unsigned long long*>(a.near_tie),
+                static_cast<unsigned long long>(__popc(ties)));
     tc_fence_before();
   }
   __syncthreads();
@@ -315,18 +481,105 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+template <bool kPredict, int kSplit>
+cudaError_t set_smem_attr(int N) {
+  return cudaFuncSetAttribute(route_tc_kernel<kPredict, kSplit>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              route_layout(N, kPredict).total);
+}
+
+template <bool kPredict, int kSplit>
+cudaError_t launch_split(const CUtensorMap& tm_h, const CUtensorMap& tm_w,
+                         const CUtensorMap& tm_wp, const RouteTcArgs& a, int tiles,
+                         cudaStream_t st, int* max_clusters) {
+  cudaError_t err = set_smem_attr<kPredict, kSplit>(a.N);
+  if (err != cudaSuccess) return err;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(tiles * kSplit);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = route_layout(a.N, kPredict).total;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kSplit;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = kSplit > 1 ? 1 : 0;
+  if (max_clusters != nullptr)  // occupancy query only
+    return cudaOccupancyMaxActiveClusters(max_clusters, route_tc_kernel<kPredict, kSplit>, &cfg);
+  return cudaLaunchKernelEx(&cfg, route_tc_kernel<kPredict, kSplit>, tm_h, tm_w, tm_wp, a);
+}
+
+template <bool kPredict>
+cudaError_t launch_any(const CUtensorMap& tm_h, const CUtensorMap& tm_w, const CUtensorMap& tm_wp,
+                       const RouteTcArgs& a, int split, int tiles, cudaStream_t st,
+                       int* max_clusters) {
+  switch (split) {
+    case 1: return launch_split<kPredict, 1>(tm_h, tm_w, tm_wp, a, tiles, st, max_clusters);
+    case 2: return launch_split<kPredict, 2>(tm_h, tm_w, tm_wp, a, tiles, st, max_clusters);
+    case 4: return launch_split<kPredict, 4>(tm_h, tm_w, tm_wp, a, tiles, st, max_clusters);
+    case 8: return launch_split<kPredict, 8>(tm_h, tm_w, tm_wp, a, tiles, st, max_clusters);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+// Clusters of `split` CTAs of this kernel that can be resident at once (0 on error), cached
+// per device and shape.
+int max_active_clusters(bool predict, int split, int N) {
+  struct Entry {
+    int dev, predict, split, N, clusters;
+  };
+  static std::mutex mu;
+  static Entry cache[64];
+  static int used = 0;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < used; ++i)
+    if (cache[i].dev == dev && cache[i].predict == (predict ? 1 : 0) &&
+        cache[i].split == split && cache[i].N == N)
+      return cache[i].clusters;
+  RouteTcArgs probe{};
+  probe.N = N;
+  CUtensorMap none{};
+  int clusters = 0;
+  const cudaError_t err =
+      predict ? launch_any<true>(none, none, none, probe, split, 1, nullptr, &clusters)
+              : launch_any<false>(none, none, none, probe, split, 1, nullptr, &clusters);
+  if (err != cudaSuccess) {
+    (void)cudaGetLastError();
+    clusters = 0;
+  }
+  if (used < 64) cache[used++] = Entry{dev, predict ? 1 : 0, split, N, clusters};
+  return clusters;
+}
+
 }  // namespace
 
+int route_split(int T, int N, int d, bool predict, int num_sms) {
+  const RouteSmemLayout L = route_layout(N, predict);
+  const int tiles = (T + kTileM - 1) / kTileM;
+  const int KB = d / kBK;
+  if (route_recv_bytes(L.b_rows) > L.stages * L.stage_bytes) return 1;
+  for (int s = kMaxSplit; s > 1; s >>= 1) {
+    if (N % s != 0 || (N / s) % 16 != 0 || KB % s != 0 || tiles * s > num_sms) continue;
+    if (max_active_clusters(predict, s, N) < tiles) continue;  // must fit in one wave
+    return s;
+  }
+  return 1;
+}
+
 cudaError_t launch_route_tc(bool predict, const CUtensorMap& tm_h, const CUtensorMap& tm_w,
-                            const CUtensorMap& tm_wp, const RouteTcArgs& a, cudaStream_t st) {
+                            const CUtensorMap& tm_wp, const RouteTcArgs& a, int split,
+                            cudaStream_t st) {
   if (a.T == 0) return cudaSuccess;
-  const RouteSmemLayout L = route_layout(a.N, predict);
-  cudaError_t err = cudaFuncSetAttribute(route_tc_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, L.total);
-  if (err != cudaSuccess) return err;
-  dim3 grid((a.T + kTileM - 1) / kTileM);
-  route_tc_kernel<<<grid, kThreads, L.total, st>>>(tm_h, tm_w, tm_wp, a, predict ? 1 : 0);
-  return cudaGetLastError();
+  if (split < 1 || split > kMaxSplit || a.N % split != 0 || (a.N / split) % 16 != 0 ||
+      (a.d / kBK) % split != 0)
+    return cudaErrorInvalidValue;
+  const int tiles = (a.T + kTileM - 1) / kTileM;
+  return predict ? launch_any<true>(tm_h, tm_w, tm_wp, a, split, tiles, st, nullptr)
+                 : launch_any<false>(tm_h, tm_w, tm_wp, a, split, tiles, st, nullptr);
 }
 
 }  // namespace pr2

@@ -122,13 +122,14 @@ def test_layer_is_deterministic():
     assert torch.equal(a["out"], b["out"]) and torch.equal(a["perm"], b["perm"])
 
 
-def test_invalid_replay_indices_are_flagged_and_skipped():
-    cfg = synth.LayerConfig("bad", T=130, d=256, N=16, k=4, m=128)
+@pytest.mark.parametrize("N", [16, 64])  # one CTA per tile; a 4-CTA cluster splitting experts
+def test_invalid_replay_indices_are_flagged_and_skipped(N):
+    cfg = synth.LayerConfig("bad", T=130, d=256, N=N, k=4, m=128)
     L = synth.make_layer(cfg, seed=2)
     Ld = H.to_dev(L)
     orc = oracle.route_predict(L["x"], L["W_router"], L["W_pred"], cfg.k)
     idx = orc["idx"].copy()
-    idx[3, 1] = 16       # out of range
+    idx[3, 1] = N        # out of range
     idx[7, 2] = -5       # negative
     idx[129, 3] = idx[129, 0]  # duplicate within the token (last, ragged tile)
     idx_d = torch.from_numpy(idx).cuda()
