@@ -197,23 +197,33 @@ def run_pr2(args, rank, world, local_rank):
         e.record()  # creates the underlying cudaEvent_t
         return e
 
+    def rec(e):
+        if e is not None:
+            e.record()
+
     def step(x, evs):
-        evs[0].record()
+        rec(evs[0])
         B.check(B.pr2_route_predict(dm, x, L["W_router"], L["W_pred"], idx, gates, logits, near,
                                     status), "pr2_route_predict")
-        evs[1].record()
+        rec(evs[1])
         B.check(B.pr2_moe_forward(dm, x, idx, gates, L["W_gate"], L["W_up"], L["W_down"],
                                   L["Ws_gate"], L["Ws_up"], L["Ws_down"], out1, workspace=ws,
                                   status=status, events=evs[2]), "pr2_moe_forward")
-        evs[3].record()
+        rec(evs[3])
         B.check(B.pr2_route_replay(dm, x, W2, idx, rgates, None, status), "pr2_route_replay")
-        evs[4].record()
+        rec(evs[4])
         B.check(B.pr2_moe_forward(dm, x, idx, rgates, L["W_gate"], L["W_up"], L["W_down"],
                                   L["Ws_gate"], L["Ws_up"], L["Ws_down"], out2, workspace=ws,
                                   status=status, events=evs[5]), "pr2_moe_forward")
-        evs[6].record()
+        rec(evs[6])
 
-    def make_evs():
+    def make_evs(stages):
+        """Step-boundary events, plus (stages=True) an event at every stage boundary.  Events
+        between kernels stop a kernel's prologue from overlapping the previous kernel's tail
+        (programmatic dependent launch), so the headline steps record step boundaries only and
+        the per-kernel breakdown comes from a separate pass."""
+        if not stages:
+            return [ev(), None, None, None, None, None, ev()]
         a = [ev() for _ in range(5)]
         b = [ev() for _ in range(5)]
         return [ev(), ev(), (B.stage_events(a), a), ev(), ev(), (B.stage_events(b), b), ev()]
@@ -223,15 +233,16 @@ def run_pr2(args, rank, world, local_rank):
             flush.fill_(i & 0xFF)
             e = evsets[i]
             step(L["x"] if x is None else x,
-                 [e[0], e[1], e[2][0], e[3], e[4], e[5][0], e[6]])
+                 [e[0], e[1], e[2][0] if e[2] else None, e[3], e[4], e[5][0] if e[5] else None,
+                  e[6]])
 
     # warm-up
-    wev = [make_evs() for _ in range(args.warmup)]
+    wev = [make_evs(False) for _ in range(args.warmup)]
     run(args.warmup, wev)
     torch.cuda.synchronize()
     if int(status.item()) != 0:
         raise RuntimeError(f"device status {int(status.item())} after warm-up")
-    evsets = [make_evs() for _ in range(args.steps)]
+    evsets = [make_evs(False) for _ in range(args.steps)]
     if dist is not None:
         dist.barrier()
     torch.cuda.synchronize()
@@ -248,9 +259,15 @@ def run_pr2(args, rank, world, local_rank):
     def el(a, b):
         return a.elapsed_time(b)  # ms
 
+    total_ms = sum(el(e[0], e[6]) for e in evsets)
+    # per-kernel breakdown: a separate pass with an event at every stage boundary
+    n_break = min(args.steps, 200)
+    bsets = [make_evs(True) for _ in range(n_break)]
+    run(n_break, bsets)
+    torch.cuda.synchronize()
     per = dict(step=[], route_predict=[], route_replay=[], dispatch=[], gate_up=[], down=[],
                combine=[], layer_rollout=[], layer_replay=[])
-    for e in evsets:
+    for e in bsets:
         per["step"].append(el(e[0], e[6]))
         per["route_predict"].append(el(e[0], e[1]))
         per["route_replay"].append(el(e[3], e[4]))
@@ -261,7 +278,6 @@ def run_pr2(args, rank, world, local_rank):
             per["gate_up"].append(el(st[1], st[2]))
             per["down"].append(el(st[2], st[3]))
             per["combine"].append(el(st[3], st[4]))
-    total_ms = sum(per["step"])
     if dist is not None:
         t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -326,8 +342,7 @@ def run_pr2(args, rank, world, local_rank):
         flush.fill_(i & 0xFF)
         a = ev()
         xd.copy_(xh, non_blocking=True)
-        e = make_evs()
-        step(xd, [e[0], e[1], e[2][0], e[3], e[4], e[5][0], e[6]])
+        step(xd, [None] * 7)
         out1h.copy_(out1, non_blocking=True)
         out2h.copy_(out2, non_blocking=True)
         idxh.copy_(idx, non_blocking=True)
@@ -352,7 +367,9 @@ def run_pr2(args, rank, world, local_rank):
                 config=workload_desc(cfg), roofline=roofline, e2e=e2e,
                 gpu_launches=launches_per_step * args.steps, clocks=clk,
                 modes=dict(rollout_tokens_per_s=cfg.T / (mean["layer_rollout"] / 1e3),
-                           replay_tokens_per_s=cfg.T / (mean["layer_replay"] / 1e3)),
+                           replay_tokens_per_s=cfg.T / (mean["layer_replay"] / 1e3),
+                           note="from the per-kernel breakdown pass (stage events)"),
+                breakdown_ms_per_step=mean["step"],
                 kernels=kernels, near_tie_tokens_per_step=near_per_step)
 
     if rank == 0 and not args.no_cpu_baseline:

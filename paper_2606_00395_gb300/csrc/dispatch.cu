@@ -37,6 +37,8 @@ __global__ void __launch_bounds__(kDispatchChunk)
                 int32_t* __restrict__ blk_hist, int32_t* status) {
   __shared__ int hist[kMaxExpertsDispatch];
   for (int e = threadIdx.x; e < N; e += blockDim.x) hist[e] = 0;
+  pdl_wait();
+  pdl_trigger();
   __syncthreads();
   const int64_t f = static_cast<int64_t>(blockIdx.x) * kDispatchChunk + threadIdx.x;
   if (f < F) {
@@ -90,6 +92,8 @@ __global__ void __launch_bounds__(1024)
   __shared__ int part[1024];  // [G][N_pad] partial sums, then their exclusive scan over g
   __shared__ int ex_off[kMaxExpertsDispatch + 1];
   __shared__ int ex_tile[kMaxExpertsDispatch + 1];
+  pdl_wait();
+  pdl_trigger();
   const int tid = threadIdx.x;
   int n_pad = 32;
   while (n_pad < N) n_pad <<= 1;
@@ -173,6 +177,8 @@ __global__ void __launch_bounds__(kDispatchChunk)
   __shared__ int wcnt[kWarps][kMaxExpertsDispatch];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int i = threadIdx.x; i < kWarps * N; i += blockDim.x) wcnt[i / N][i % N] = 0;
+  pdl_wait();
+  pdl_trigger();
   __syncthreads();
   const int64_t f = static_cast<int64_t>(blockIdx.x) * kDispatchChunk + threadIdx.x;
   int e = -1;
@@ -206,6 +212,8 @@ __global__ void __launch_bounds__(256)
     gather_kernel(const uint4* __restrict__ h, const int32_t* __restrict__ perm,
                   const int32_t* __restrict__ nrows_ptr, int k, int row_vec,
                   uint4* __restrict__ X) {
+  pdl_wait();
+  pdl_trigger();
   const int nrows = *nrows_ptr;
   const int lane = threadIdx.x & 31;
   const int warp0 = static_cast<int>((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
@@ -224,6 +232,8 @@ __global__ void __launch_bounds__(256)
     combine_kernel(const T* __restrict__ Y, const T* __restrict__ Ys,
                    const int32_t* __restrict__ inv, const float* __restrict__ gates, int64_t Tn,
                    int k, int d, int n_shared, T* __restrict__ out) {
+  pdl_wait();
+  pdl_trigger();
   const int lane = threadIdx.x & 31;
   const int64_t warp0 = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
@@ -281,23 +291,30 @@ cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st)
   const int64_t F = a.T * a.k;
   const int nblk = static_cast<int>((F + kDispatchChunk - 1) / kDispatchChunk);
   if (nblk > 0) {
-    hist_kernel<<<nblk, kDispatchChunk, 0, st>>>(a.idx, F, a.k, a.N, a.blk_hist, a.status);
+    cudaError_t err = launch_pdl(hist_kernel, dim3(nblk), dim3(kDispatchChunk), 0, st, 1,
+                                 a.idx, F, a.k, a.N, a.blk_hist, a.status);
+    if (err != cudaSuccess) return err;
   }
-  scan_kernel<<<1, 1024, 0, st>>>(a.blk_hist, nblk, a.N, a.T, a.n_shared, a.counts, a.offsets,
-                                  a.tiles, a.num_tiles, a.stiles1, a.stiles2);
+  cudaError_t err = launch_pdl(scan_kernel, dim3(1), dim3(1024), 0, st, 1, a.blk_hist, nblk, a.N,
+                               a.T, a.n_shared, a.counts, a.offsets, a.tiles, a.num_tiles,
+                               a.stiles1, a.stiles2);
+  if (err != cudaSuccess) return err;
   if (nblk > 0) {
-    place_kernel<<<nblk, kDispatchChunk, 0, st>>>(a.idx, F, a.k, a.N, a.blk_hist, a.perm,
-                                                  a.inv);
+    err = launch_pdl(place_kernel, dim3(nblk), dim3(kDispatchChunk), 0, st, 1, a.idx, F, a.k,
+                     a.N, static_cast<const int32_t*>(a.blk_hist), a.perm, a.inv);
+    if (err != cudaSuccess) return err;
     const int row_vec = a.d * a.esz / 16;
     int64_t warps_needed = F;
     int64_t blocks = (warps_needed + 7) / 8;
     const int64_t cap = static_cast<int64_t>(num_sms) * 8;
     if (blocks > cap) blocks = cap;
-    gather_kernel<<<static_cast<int>(blocks), 256, 0, st>>>(
-        static_cast<const uint4*>(a.h), a.perm, a.offsets + a.N, a.k, row_vec,
-        static_cast<uint4*>(a.xperm));
+    err = launch_pdl(gather_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, 1,
+                     static_cast<const uint4*>(a.h), static_cast<const int32_t*>(a.perm),
+                     static_cast<const int32_t*>(a.offsets + a.N), a.k, row_vec,
+                     static_cast<uint4*>(a.xperm));
+    if (err != cudaSuccess) return err;
   }
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st) {
@@ -305,24 +322,23 @@ cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st) {
   int64_t blocks = (a.T + 7) / 8;
   const int64_t cap = static_cast<int64_t>(num_sms) * 8;
   if (blocks > cap) blocks = cap;
-  if (a.bf16 && a.k <= 8) {
-    combine_kernel<__nv_bfloat16, 8, 8><<<static_cast<int>(blocks), 256, 0, st>>>(
-        static_cast<const __nv_bfloat16*>(a.Y), static_cast<const __nv_bfloat16*>(a.Ys), a.inv,
-        a.gates, a.T, a.k, a.d, a.n_shared, static_cast<__nv_bfloat16*>(a.out));
-  } else if (a.bf16) {
-    combine_kernel<__nv_bfloat16, 8, 32><<<static_cast<int>(blocks), 256, 0, st>>>(
-        static_cast<const __nv_bfloat16*>(a.Y), static_cast<const __nv_bfloat16*>(a.Ys), a.inv,
-        a.gates, a.T, a.k, a.d, a.n_shared, static_cast<__nv_bfloat16*>(a.out));
-  } else if (a.k <= 8) {
-    combine_kernel<float, 4, 8><<<static_cast<int>(blocks), 256, 0, st>>>(
-        static_cast<const float*>(a.Y), static_cast<const float*>(a.Ys), a.inv, a.gates, a.T,
-        a.k, a.d, a.n_shared, static_cast<float*>(a.out));
-  } else {
-    combine_kernel<float, 4, 32><<<static_cast<int>(blocks), 256, 0, st>>>(
-        static_cast<const float*>(a.Y), static_cast<const float*>(a.Ys), a.inv, a.gates, a.T,
-        a.k, a.d, a.n_shared, static_cast<float*>(a.out));
+  const dim3 grid(static_cast<unsigned>(blocks)), block(256);
+  if (a.bf16) {
+    auto* Y = static_cast<const __nv_bfloat16*>(a.Y);
+    auto* Ys = static_cast<const __nv_bfloat16*>(a.Ys);
+    auto* out = static_cast<__nv_bfloat16*>(a.out);
+    return a.k <= 8 ? launch_pdl(combine_kernel<__nv_bfloat16, 8, 8>, grid, block, 0, st, 1, Y,
+                                 Ys, a.inv, a.gates, a.T, a.k, a.d, a.n_shared, out)
+                    : launch_pdl(combine_kernel<__nv_bfloat16, 8, 32>, grid, block, 0, st, 1, Y,
+                                 Ys, a.inv, a.gates, a.T, a.k, a.d, a.n_shared, out);
   }
-  return cudaGetLastError();
+  auto* Y = static_cast<const float*>(a.Y);
+  auto* Ys = static_cast<const float*>(a.Ys);
+  auto* out = static_cast<float*>(a.out);
+  return a.k <= 8 ? launch_pdl(combine_kernel<float, 4, 8>, grid, block, 0, st, 1, Y, Ys, a.inv,
+                               a.gates, a.T, a.k, a.d, a.n_shared, out)
+                  : launch_pdl(combine_kernel<float, 4, 32>, grid, block, 0, st, 1, Y, Ys, a.inv,
+                               a.gates, a.T, a.k, a.d, a.n_shared, out);
 }
 
 }  // namespace pr2

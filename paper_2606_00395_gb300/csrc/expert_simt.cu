@@ -17,6 +17,8 @@ __global__ void __launch_bounds__(kCols)
                        const float* __restrict__ W1, const TileEntry* __restrict__ tiles,
                        const int32_t* __restrict__ num_tiles, int K, int n_out, int b_rows,
                        float* __restrict__ out) {
+  pdl_wait();
+  pdl_trigger();
   if (static_cast<int>(blockIdx.x) >= *num_tiles) return;
   const TileEntry te = tiles[blockIdx.x];
   const int c = blockIdx.y * kCols + threadIdx.x;
@@ -45,10 +47,9 @@ cudaError_t launch_expert_simt(bool swiglu, const float* A, const float* Wb0, co
                                const GemmArgs& g, cudaStream_t st) {
   if (g.max_tiles <= 0) return cudaSuccess;
   dim3 grid(g.max_tiles, (g.n_out + kCols - 1) / kCols);
-  expert_simt_kernel<<<grid, kCols, 0, st>>>(swiglu ? 1 : 0, A, Wb0, Wb1, g.tiles, g.num_tiles,
-                                             g.K, g.n_out, g.b_rows_per_expert,
-                                             static_cast<float*>(g.out));
-  return cudaGetLastError();
+  return launch_pdl(expert_simt_kernel, grid, dim3(kCols), 0, st, 1, swiglu ? 1 : 0, A, Wb0, Wb1,
+                    static_cast<const TileEntry*>(g.tiles), g.num_tiles, g.K, g.n_out,
+                    g.b_rows_per_expert, static_cast<float*>(g.out));
 }
 
 }  // namespace pr2

@@ -49,7 +49,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int lane = threadIdx.x & 31;
   constexpr int kColsPerTile = kSwiGLU ? kBN / 2 : kBN;  // output columns per N-tile
   const int n_tiles_n = (g.n_out + kColsPerTile - 1) / kColsPerTile;
-  const int num_tiles = (*g.num_tiles) * n_tiles_n;
   const int KB = g.K / kBK;
 
   if (threadIdx.x == 0) {
@@ -75,6 +74,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_wait();  // the tile table and the A operand come from the previous kernels
+  pdl_trigger();
+  const int num_tiles = (*g.num_tiles) * n_tiles_n;
 
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer ----------------
@@ -236,19 +238,11 @@ cudaError_t launch_expert_tc(bool swiglu, const CUtensorMap& tm_a, const CUtenso
   const int cols = swiglu ? kBN / 2 : kBN;
   const int64_t bound = static_cast<int64_t>(g.max_tiles) * ((g.n_out + cols - 1) / cols);
   const int grid = static_cast<int>(bound < num_sms ? bound : num_sms);
-  cudaError_t err;
-  if (swiglu) {
-    err = cudaFuncSetAttribute(expert_tc_kernel<true>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-    if (err != cudaSuccess) return err;
-    expert_tc_kernel<true><<<grid, kThreads, kSmemBytes, st>>>(tm_a, tm_b0, tm_b1, g);
-  } else {
-    err = cudaFuncSetAttribute(expert_tc_kernel<false>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-    if (err != cudaSuccess) return err;
-    expert_tc_kernel<false><<<grid, kThreads, kSmemBytes, st>>>(tm_a, tm_b0, tm_b1, g);
-  }
-  return cudaGetLastError();
+  auto* kernel = swiglu ? expert_tc_kernel<true> : expert_tc_kernel<false>;
+  const cudaError_t err =
+      cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+  if (err != cudaSuccess) return err;
+  return launch_pdl(kernel, dim3(grid), dim3(kThreads), kSmemBytes, st, 1, tm_a, tm_b0, tm_b1, g);
 }
 
 }  // namespace pr2

@@ -26,6 +26,18 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   return t;
 }
 
+// Programmatic dependent launch.  Every kernel of the library is launched with programmatic
+// stream serialization, so its prologue (barrier init, TMEM allocation, descriptor prefetch) can
+// overlap the tail of the previous kernel in the stream.  pdl_wait() returns once the kernels
+// this grid depends on have completed and their memory is visible (at once when there are
+// none); no global memory is touched before it.  pdl_trigger() lets the next kernel start its
+// prologue once every CTA of this grid has triggered or exited; that kernel still waits for
+// this one to complete before it touches memory.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

@@ -18,6 +18,8 @@ __global__ void __launch_bounds__(kWarps * 32)
                       const int32_t* __restrict__ idx_in, int32_t* __restrict__ idx_out,
                       float* __restrict__ gates, float* __restrict__ aux,
                       unsigned long long* near_tie, int32_t* status) {
+  pdl_wait();
+  pdl_trigger();
   const int lane = threadIdx.x & 31;
   const int t = blockIdx.x * kWarps + (threadIdx.x >> 5);
   if (t >= T) return;
@@ -66,10 +68,9 @@ cudaError_t launch_route_simt(const pr2_dims& dm, bool predict, const float* h, 
   const int T = static_cast<int>(dm.T);
   if (T == 0) return cudaSuccess;
   dim3 grid((T + kWarps - 1) / kWarps);
-  route_simt_kernel<<<grid, kWarps * 32, 0, st>>>(
-      T, dm.d, dm.N, dm.k, predict ? 1 : 0, h, W, Wp, idx_in, idx_out, gates, aux,
-      reinterpret_cast<unsigned long long*>(near_tie), status);
-  return cudaGetLastError();
+  return launch_pdl(route_simt_kernel, grid, dim3(kWarps * 32), 0, st, 1, T, dm.d, dm.N, dm.k,
+                    predict ? 1 : 0, h, W, Wp, idx_in, idx_out, gates, aux,
+                    reinterpret_cast<unsigned long long*>(near_tie), status);
 }
 
 }  // namespace pr2

@@ -199,6 +199,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_wait();  // h, the weights and the cached route may come from the previous kernels
+  pdl_trigger();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -494,21 +496,23 @@ cudaError_t launch_split(const CUtensorMap& tm_h, const CUtensorMap& tm_w,
                          cudaStream_t st, int* max_clusters) {
   cudaError_t err = set_smem_attr<kPredict, kSplit>(a.N);
   if (err != cudaSuccess) return err;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(tiles * kSplit);
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = route_layout(a.N, kPredict).total;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = kSplit;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = kSplit > 1 ? 1 : 0;
-  if (max_clusters != nullptr)  // occupancy query only
+  const size_t smem = route_layout(a.N, kPredict).total;
+  if (max_clusters != nullptr) {  // occupancy query only
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(tiles * kSplit);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = kSplit;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
     return cudaOccupancyMaxActiveClusters(max_clusters, route_tc_kernel<kPredict, kSplit>, &cfg);
-  return cudaLaunchKernelEx(&cfg, route_tc_kernel<kPredict, kSplit>, tm_h, tm_w, tm_wp, a);
+  }
+  return launch_pdl(route_tc_kernel<kPredict, kSplit>, dim3(tiles * kSplit), dim3(kThreads), smem,
+                    st, kSplit, tm_h, tm_w, tm_wp, a);
 }
 
 template <bool kPredict>
