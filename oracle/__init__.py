@@ -11,6 +11,10 @@ Functions (each cites the passage it follows in the C source):
 * ``route_replay``   - Sec. 4.1 "Replay During Training" (Algorithm 1 replay steps, Algorithm 3)
 * ``permute``        - dispatch to experts as a stable counting sort (Algorithm 1)
 * ``moe_forward``    - Eqs. pr2_old_output / pr2_output with SwiGLU experts (App. E.2)
+* ``predictor_loss`` - Eq. pr2_loss and Algorithm 3 (loss and W_p gradient), and the
+  delta-matching variant of the appendix ablation
+* ``route_diagnostics`` - top-k agreement and the deviation histogram (Sec. 5)
+* ``feature_cache``  - the fixed-length feature cache of Algorithm 2 (evenly spaced positions)
 
 Parity status: every function is pinned by the CPU tests in ``tests/test_oracle_pins.py``.
 """
@@ -62,6 +66,12 @@ def bind(path: str):
     lib.oracle_moe_forward.argtypes = [I64, P, I64, I32, I32, I32, I32, I32, I32, P, P, P, P,
                                        P, P, P, P, P, P]
     lib.oracle_moe_forward.restype = None
+    lib.oracle_predictor_loss.argtypes = [I64, I32, I32, I32, I32, P, P, P, P, I64, P, P, P, P]
+    lib.oracle_predictor_loss.restype = I64
+    lib.oracle_route_diagnostics.argtypes = [I64, I32, I32, P, P, P]
+    lib.oracle_route_diagnostics.restype = I64
+    lib.oracle_feature_cache.argtypes = [I64, I64, I32, I32, I32, P, P, P, P, P]
+    lib.oracle_feature_cache.restype = None
     lib.oracle_num_threads.argtypes = []
     lib.oracle_num_threads.restype = I32
     return lib
@@ -190,3 +200,76 @@ def moe_forward(h, idx, gates, W_gate, W_up, W_down, Ws_gate=None, Ws_up=None, W
                                _ptr(gt), _ptr(g), _ptr(u), _ptr(dn), _ptr(sg), _ptr(su), _ptr(sd),
                                _ptr(out))
     return out
+
+
+def _f32(a) -> np.ndarray:
+    """fp32 contiguous numpy copy of a tensor / array that is stored as fp32."""
+    if isinstance(a, torch.Tensor):
+        if a.dtype != torch.float32:
+            raise TypeError(f"expected an fp32 tensor, got {a.dtype}")
+        return a.detach().to("cpu").contiguous().numpy()
+    a = np.ascontiguousarray(a)
+    if a.dtype != np.float32:
+        raise TypeError(f"expected fp32, got {a.dtype}")
+    return a
+
+
+def predictor_loss(h_old, p_old, W_pred, rho, pos=None, delta: bool = False, lib=None):
+    """Eq. pr2_loss for one layer (``delta``: the delta-matching variant) in fp64.
+
+    h_old [T_c,d] (fp32 or bf16), p_old [T_c,N] fp32, W_pred [N,d] (h_old's dtype), rho
+    [T_rho,N] fp32 teacher probabilities, pos [T_c] int32 rows of rho (None: row c).  Returns
+    dict(loss, kl [T_c], grad [N,d], bad = #invalid pos)."""
+    hs, c0 = _stored(h_old)
+    ws, c1 = _stored(W_pred)
+    dt = _same_dtype(c0, c1)
+    po = _f32(p_old)
+    rh = _f32(rho)
+    Tc, d = hs.shape
+    N = ws.shape[0]
+    ps = None if pos is None else np.ascontiguousarray(np.asarray(pos, dtype=np.int32))
+    loss = np.zeros(1)
+    kl = np.zeros(max(Tc, 1))
+    grad = np.zeros((N, d))
+    bad = _load(lib).oracle_predictor_loss(Tc, d, N, dt, 1 if delta else 0, _ptr(hs), _ptr(po),
+                                           _ptr(ws), _ptr(rh), rh.shape[0], _ptr(ps),
+                                           _ptr(loss), _ptr(kl), _ptr(grad))
+    return dict(loss=float(loss[0]), kl=kl[:Tc], grad=grad, bad=int(bad))
+
+
+def route_diagnostics(rho, idx_cached, lib=None):
+    """Top-k agreement and deviation histogram of a cached route against TopK(rho, k).
+    Returns dict(hist [k+1] int64, overlap = sum_t |Î_t ∩ I_t|, agreement = overlap / (T k))."""
+    rh = _f32(rho)
+    ix = np.ascontiguousarray(np.asarray(idx_cached, dtype=np.int32))
+    T, N = rh.shape
+    k = ix.shape[1]
+    hist = np.zeros(k + 1, np.int64)
+    ov = _load(lib).oracle_route_diagnostics(T, N, k, _ptr(rh), _ptr(ix), _ptr(hist))
+    return dict(hist=hist, overlap=int(ov), agreement=(ov / (T * k)) if T else 0.0)
+
+
+def feature_cache(h, logits, Tc: int, lib=None):
+    """Feature-cache rows of Algorithm 2 at evenly spaced positions: dict(pos [T_c] int32,
+    h [T_c,d] (h's dtype), p [T_c,N] fp32)."""
+    if isinstance(h, torch.Tensor):
+        ht = h.detach().to("cpu").contiguous()
+        esz = ht.element_size()
+        raw = ht.view(torch.int16 if esz == 2 else torch.int32).numpy()
+    else:
+        raw = np.ascontiguousarray(h)
+        esz = raw.dtype.itemsize
+    lg = _f32(logits)
+    T, d = raw.shape
+    N = lg.shape[1]
+    if not (0 <= Tc <= T):
+        raise ValueError("need 0 <= T_c <= T")
+    pos = np.zeros(max(Tc, 1), np.int32)
+    ch = np.zeros((max(Tc, 1), d), raw.dtype)
+    cp = np.zeros((max(Tc, 1), N), np.float32)
+    _load(lib).oracle_feature_cache(T, Tc, d, N, esz, _ptr(raw), _ptr(lg), _ptr(pos), _ptr(ch),
+                                    _ptr(cp))
+    hc = torch.from_numpy(ch[:Tc].copy())
+    if isinstance(h, torch.Tensor):
+        hc = hc.view(h.dtype)
+    return dict(pos=pos[:Tc], h=hc, p=cp[:Tc])

@@ -253,3 +253,158 @@ void oracle_moe_forward(int64_t n_tok, const int64_t* tokens, int64_t T, int d, 
         free(a); free(y);
     }
 }
+
+/* ---- Sec. 4.2 "Predictive Loss" (Eq. pr2_loss) and Algorithm 3 ---------------------------- */
+
+/* log Softmax(v)_j = v_j - max - log sum_i exp(v_i - max) for finite v_j; entries equal to
+ * -inf get -inf.  Writes the probabilities to `pr` and their logs to `lg`. */
+static void log_softmax(const double* v, int N, double* pr, double* lg) {
+    double mx = -INFINITY;
+    for (int j = 0; j < N; ++j) if (v[j] > mx) mx = v[j];
+    double s = 0.0;
+    for (int j = 0; j < N; ++j) s += (v[j] == -INFINITY) ? 0.0 : exp(v[j] - mx);
+    double ls = log(s);
+    for (int j = 0; j < N; ++j) {
+        lg[j] = (v[j] == -INFINITY) ? -INFINITY : v[j] - mx - ls;
+        pr[j] = (v[j] == -INFINITY) ? 0.0 : exp(lg[j]);
+    }
+}
+
+/*
+ * Predictive loss of one layer over the T_c cached tokens and its gradient w.r.t. W_p.
+ * Cached route-recording features (Algorithm 2, feature cache F): h_old[T_c,d] in the stored
+ * dtype and p_old[T_c,N] fp32.  Teacher (stop-gradient): the current routing distribution
+ * rho = Softmax(h W) (Algorithm 3, first step) of the token each cached row belongs to, row
+ * pos[c] of rho_full[T_rho,N] (fp32; pos NULL means row c).
+ *
+ * kind 0, Eq. pr2_loss / Algorithm 3 ("reconstruct", "KL"):
+ *   z = p_old + h_old W_p^T,  rho_hat = Softmax(z),
+ *   KL_c = sum_j rho_j (log rho_j - log rho_hat_j)   (terms with rho_j = 0 are 0),
+ *   dKL_c / dz_j = rho_hat_j - rho_j                  (softmax Jacobian, sum_j rho_j = 1).
+ * kind 1, the delta-matching alternative (App. "Predictive Objective Ablation"):
+ *   target q = Softmax(Delta p), Delta p = p - p_old.  The teacher is given as probabilities,
+ *   and Softmax(log rho - p_old) = Softmax(p - logsumexp(p) - p_old) = Softmax(Delta p);
+ *   prediction Softmax(b), b = h_old W_p^T;  KL_c = KL(q || Softmax(b)),
+ *   dKL_c / db_j = Softmax(b)_j - q_j.
+ * loss = (1/T_c) sum_c KL_c  (the expectation over cached tokens of Eq. pr2_loss, one layer);
+ * grad[j*d + i] = (1/T_c) sum_c dKL_c/dz_j h_old[c,i]  (b_j = sum_i h_old[c,i] W_p[j*d + i]).
+ * A pos entry outside [0, T_rho) is invalid: that row contributes nothing and is counted in
+ * the return value.  kl_tok[T_c] may be NULL.  T_c = 0 gives loss 0 and a zero gradient.
+ */
+int64_t oracle_predictor_loss(int64_t Tc, int d, int N, int dtype, int kind, const void* h_old,
+                              const float* p_old, const void* Wp, const float* rho_full,
+                              int64_t T_rho, const int32_t* pos, double* loss, double* kl_tok,
+                              double* grad) {
+    double* dz = (double*)calloc((size_t)(Tc > 0 ? Tc : 1) * (size_t)N, sizeof(double));
+    double* kl = (double*)calloc((size_t)(Tc > 0 ? Tc : 1), sizeof(double));
+    int64_t bad = 0;
+    #pragma omp parallel reduction(+ : bad)
+    {
+        double* b = (double*)malloc(sizeof(double) * (size_t)N);
+        double* v = (double*)malloc(sizeof(double) * (size_t)N);
+        double* tgt = (double*)malloc(sizeof(double) * (size_t)N);
+        double* ltgt = (double*)malloc(sizeof(double) * (size_t)N);
+        double* pred = (double*)malloc(sizeof(double) * (size_t)N);
+        double* lpred = (double*)malloc(sizeof(double) * (size_t)N);
+        #pragma omp for schedule(dynamic, 4)
+        for (int64_t c = 0; c < Tc; ++c) {
+            int64_t r = pos ? (int64_t)pos[c] : c;
+            if (r < 0 || r >= T_rho) { bad += 1; continue; }
+            project(h_old, c, d, N, Wp, dtype, b);              /* b = h_old W_p */
+            const float* rho = rho_full + r * (int64_t)N;
+            const float* po = p_old + c * (int64_t)N;
+            if (kind == 0) {
+                for (int j = 0; j < N; ++j) {
+                    tgt[j] = (double)rho[j];
+                    ltgt[j] = (rho[j] > 0.0f) ? log((double)rho[j]) : -INFINITY;
+                    v[j] = (double)po[j] + b[j];                    /* z = p_old + b */
+                }
+                log_softmax(v, N, pred, lpred);                     /* rho_hat */
+            } else {
+                for (int j = 0; j < N; ++j)
+                    v[j] = (rho[j] > 0.0f) ? log((double)rho[j]) - (double)po[j] : -INFINITY;
+                log_softmax(v, N, tgt, ltgt);                       /* q = Softmax(Delta p) */
+                log_softmax(b, N, pred, lpred);                     /* Softmax(b) */
+            }
+            double acc = 0.0;
+            for (int j = 0; j < N; ++j) {
+                if (tgt[j] > 0.0) acc += tgt[j] * (ltgt[j] - lpred[j]);
+                dz[c * N + j] = pred[j] - tgt[j];
+            }
+            kl[c] = acc;
+        }
+        free(b); free(v); free(tgt); free(ltgt); free(pred); free(lpred);
+    }
+    double tot = 0.0;
+    for (int64_t c = 0; c < Tc; ++c) tot += kl[c];
+    *loss = (Tc > 0) ? tot / (double)Tc : 0.0;
+    if (kl_tok) for (int64_t c = 0; c < Tc; ++c) kl_tok[c] = kl[c];
+    #pragma omp parallel for schedule(static)
+    for (int j = 0; j < N; ++j)
+        for (int i = 0; i < d; ++i) {
+            double acc = 0.0;
+            for (int64_t c = 0; c < Tc; ++c)
+                acc += dz[c * N + j] * widen(h_old, c * (int64_t)d + i, dtype);
+            grad[(int64_t)j * d + i] = (Tc > 0) ? acc / (double)Tc : 0.0;
+        }
+    free(dz); free(kl);
+    return bad;
+}
+
+/* ---- Sec. 5 "Top-k Agreement and Route KL", "Deviation Tails" ----------------------------- */
+
+/*
+ * Route tracking of a cached route against the current router.  I_t = TopK(rho_t, k) of the
+ * current routing distribution (rho[T,N] fp32 as stored, exact in double; ties to the lower
+ * expert, as in Eq. pr2_route), Î_t = idx_cached[t].  overlap_t = |Î_t ∩ I_t|, where an entry
+ * outside [0,N) or repeated within its token never matches.  hist[k - overlap_t] += 1 (the
+ * deviation count of "Deviation Tails", 0..k); returns sum_t overlap_t, so the top-k agreement
+ * averaged over tokens is that sum / (T k).
+ */
+int64_t oracle_route_diagnostics(int64_t T, int N, int k, const float* rho,
+                                 const int32_t* idx_cached, int64_t* hist) {
+    for (int c = 0; c <= k; ++c) hist[c] = 0;
+    int64_t total = 0;
+    double* r = (double*)malloc(sizeof(double) * (size_t)N);
+    double* tv = (double*)malloc(sizeof(double) * (size_t)(k + 1));
+    int32_t* sel = (int32_t*)malloc(sizeof(int32_t) * (size_t)k);
+    char* taken = (char*)malloc((size_t)N);
+    for (int64_t t = 0; t < T; ++t) {
+        for (int j = 0; j < N; ++j) r[j] = (double)rho[t * (int64_t)N + j];
+        topk(r, N, k, sel, tv, taken);                 /* sets taken[e] for the k+1 best */
+        memset(taken, 0, (size_t)N);
+        for (int s = 0; s < k; ++s) taken[sel[s]] = 1;  /* keep exactly I_t */
+        int ov = 0;
+        for (int s = 0; s < k; ++s) {
+            int32_t e = idx_cached[t * k + s];
+            int ok = (e >= 0 && e < N);
+            for (int s2 = 0; ok && s2 < s; ++s2) if (idx_cached[t * k + s2] == e) ok = 0;
+            if (ok && taken[e]) ++ov;
+        }
+        hist[k - ov] += 1;
+        total += ov;
+    }
+    free(r); free(tv); free(sel); free(taken);
+    return total;
+}
+
+/* ---- Algorithm 2 feature cache, App. "uniform sub-sampling" --------------------------------- */
+
+/*
+ * Feature-cache writer: store the route-recording features (h_old, p_old) of the T_c retained
+ * positions of a T-token rollout (Algorithm 2: "store route-recording features when (tau,l) is
+ * retained by the fixed-length feature cache").  Reading of "drawn by uniform sub-sampling along
+ * the rollout": evenly spaced positions pos_c = floor(c T / T_c), c < T_c <= T, so the whole
+ * rollout is covered (T_c = T keeps every token).  cache_h[c] = h[pos_c] (esz-byte elements,
+ * bits copied), cache_p[c] = logits[pos_c] (fp32).
+ */
+void oracle_feature_cache(int64_t T, int64_t Tc, int d, int N, int esz, const void* h,
+                          const float* logits, int32_t* pos, void* cache_h, float* cache_p) {
+    for (int64_t c = 0; c < Tc; ++c) {
+        int64_t p = (c * T) / Tc;
+        pos[c] = (int32_t)p;
+        memcpy((char*)cache_h + c * (int64_t)d * esz, (const char*)h + p * (int64_t)d * esz,
+               (size_t)d * (size_t)esz);
+        memcpy(cache_p + c * (int64_t)N, logits + p * (int64_t)N, sizeof(float) * (size_t)N);
+    }
+}

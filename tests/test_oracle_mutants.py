@@ -35,6 +35,19 @@ MUTANTS = [
     ("shared_dropped", "for (int c = 0; c < d; ++c) o[c] += y[c];", "(void)y;", 0),
     ("forward_gate_slot0", "o[c] += gates[t * k + s] * y[c];", "o[c] += gates[t * k] * y[c];", 0),
     ("bf16_widen_shift", "<< 16;", "<< 15;", 0),
+    ("loss_grad_sign", "dz[c * N + j] = pred[j] - tgt[j];", "dz[c * N + j] = tgt[j] - pred[j];", 0),
+    ("loss_kl_reversed", "if (tgt[j] > 0.0) acc += tgt[j] * (ltgt[j] - lpred[j]);",
+     "if (pred[j] > 0.0) acc += pred[j] * (lpred[j] - ltgt[j]);", 0),
+    ("loss_not_averaged", "*loss = (Tc > 0) ? tot / (double)Tc : 0.0;", "*loss = tot;", 0),
+    ("loss_grad_transposed", "grad[(int64_t)j * d + i] = ", "grad[(int64_t)i * N + j] = ", 0),
+    ("loss_predictor_dropped", "v[j] = (double)po[j] + b[j];", "v[j] = (double)po[j];", 0),
+    ("delta_target_sign", "log((double)rho[j]) - (double)po[j]", "log((double)rho[j]) + (double)po[j]", 0),
+    ("delta_predicts_with_p_old", "log_softmax(b, N, pred, lpred);", "for (int j = 0; j < N; ++j) v[j] = (double)po[j] + b[j];\n                log_softmax(v, N, pred, lpred);", 0),
+    ("loss_pos_ignored", "int64_t r = pos ? (int64_t)pos[c] : c;", "int64_t r = c;", 0),
+    ("diag_duplicates_counted", "for (int s2 = 0; ok && s2 < s; ++s2) if (idx_cached[t * k + s2] == e) ok = 0;", "", 0),
+    ("diag_hist_by_overlap", "hist[k - ov] += 1;", "hist[ov] += 1;", 0),
+    ("diag_keeps_k_plus_one", "for (int s = 0; s < k; ++s) taken[sel[s]] = 1;", "topk(r, N, k, sel, tv, taken);", 0),
+    ("cache_positions_rounded_up", "int64_t p = (c * T) / Tc;", "int64_t p = (c * T + Tc - 1) / Tc;", 0),
 ]
 
 

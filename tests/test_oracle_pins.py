@@ -295,3 +295,159 @@ def test_token_subset_matches_full_run_and_bf16_inputs_widen_exactly():
     # bf16 -> double widening is exact: same values given as fp32 give identical results
     r32 = oracle.route_predict(L["x"].float(), L["W_router"].float(), L["W_pred"].float(), 2)
     assert np.array_equal(r32["logits"], r["logits"]) and np.array_equal(r32["idx"], r["idx"])
+
+
+# ---- Eq. pr2_loss / Algorithm 3: predictive loss and its W_p gradient ----------------------
+
+def _loss_inputs(Tc=5, d=6, N=4, seed=7):
+    g = torch.Generator().manual_seed(seed)
+    # W_p on a 2^-10 grid: the +-2^-8 and +-2^-9 finite-difference steps are exact in fp32
+    Wp = torch.randint(-64, 65, (N, d), generator=g).float() / 1024
+    h = torch.randn(Tc, d, generator=g)
+    p_old = torch.randn(Tc, N, generator=g)
+    rho = torch.softmax(torch.randn(Tc, N, generator=g).double(), -1).float()
+    return h, p_old, Wp, rho
+
+
+def _dyadic_rho(T, N, g):
+    """Teacher rows on a 2^-10 grid summing to exactly 1 (in fp32 and in double)."""
+    c = torch.randint(1, 1024 // N, (T, N), generator=g)
+    c[:, -1] = 1024 - c[:, :-1].sum(1)
+    return (c.double() / 1024).float()
+
+
+@pytest.mark.parametrize("delta", [False, True])
+def test_loss_gradient_matches_finite_differences(delta):
+    h, p_old, Wp, rho = _loss_inputs()
+    r = oracle.predictor_loss(h, p_old, Wp, rho, delta=delta)
+    N, d = Wp.shape
+    eps = 2.0 ** -8
+    fd = np.zeros((N, d))
+    for j in range(N):
+        for i in range(d):
+            def L(e):
+                W = Wp.clone()
+                W[j, i] += e
+                return oracle.predictor_loss(h, p_old, W, rho, delta=delta)["loss"]
+            d1 = (L(eps) - L(-eps)) / (2 * eps)
+            d2 = (L(eps / 2) - L(-eps / 2)) / eps
+            fd[j, i] = (4 * d2 - d1) / 3  # Richardson: O(eps^4)
+    assert np.max(np.abs(fd - r["grad"])) <= 1e-7 * max(1.0, np.max(np.abs(r["grad"])))
+    assert r["loss"] > 0 and np.all(r["kl"] >= 0)
+
+
+@pytest.mark.parametrize("delta", [False, True])
+def test_loss_vanishes_at_the_teacher(delta):
+    """Teacher rho = Softmax(p_old + h W*^T): the standard loss is 0 at W_p = W*; the delta
+    target Softmax(log rho - p_old) = Softmax(h W*^T) is matched by Softmax(b) at W_p = W* too."""
+    h, p_old, Wp, _ = _loss_inputs(Tc=7, d=8, N=5, seed=3)
+    z = p_old.double() + h.double() @ Wp.double().T
+    rho = torch.softmax(z, -1).float()
+    r = oracle.predictor_loss(h, p_old, Wp, rho, delta=delta)
+    # only the fp32 rounding of rho remains: its rows sum to 1 within ~1e-7
+    assert abs(r["loss"]) < 1e-7
+    assert np.max(np.abs(r["grad"])) < 1e-6
+    other = oracle.predictor_loss(h, p_old, torch.zeros_like(Wp), rho, delta=delta)
+    assert other["loss"] > 1e-4
+
+
+def test_loss_two_experts_closed_form():
+    """N = 2: KL of two Bernoulli laws, q = sigmoid(z_1 - z_0)."""
+    h, p_old, Wp, _ = _loss_inputs(Tc=6, d=5, N=2, seed=11)
+    rho = _dyadic_rho(6, 2, torch.Generator().manual_seed(1))
+    r = oracle.predictor_loss(h, p_old, Wp, rho)
+    z = p_old.double().numpy() + h.double().numpy() @ Wp.double().numpy().T
+    q = 1.0 / (1.0 + np.exp(-(z[:, 1] - z[:, 0])))
+    a = rho.double().numpy()[:, 1]
+    kl = a * np.log(a / q) + (1 - a) * np.log((1 - a) / (1 - q))
+    assert np.max(np.abs(r["kl"] - kl)) <= 1e-12
+    assert abs(r["loss"] - kl.mean()) <= 1e-12
+
+
+def test_loss_shift_invariance_and_delta_equals_standard_at_zero_p_old():
+    h, _, Wp, _ = _loss_inputs(Tc=6, d=7, N=5, seed=5)
+    g = torch.Generator().manual_seed(2)
+    rho = _dyadic_rho(6, 5, g)
+    p_old = torch.randint(-128, 128, (6, 5), generator=g).float() / 64  # exact +2 shifts
+    a = oracle.predictor_loss(h, p_old, Wp, rho)
+    b = oracle.predictor_loss(h, p_old + 2.0, Wp, rho)
+    assert abs(a["loss"] - b["loss"]) <= 1e-12
+    assert np.max(np.abs(a["grad"] - b["grad"])) <= 1e-12
+    z = torch.zeros_like(p_old)
+    s = oracle.predictor_loss(h, z, Wp, rho)
+    t = oracle.predictor_loss(h, z, Wp, rho, delta=True)
+    assert abs(s["loss"] - t["loss"]) <= 1e-12
+    assert np.max(np.abs(s["grad"] - t["grad"])) <= 1e-12
+
+
+def test_loss_rows_follow_pos_and_invalid_rows_are_skipped():
+    h, p_old, Wp, rho = _loss_inputs(Tc=4, d=5, N=3, seed=9)
+    g = torch.Generator().manual_seed(4)
+    full = torch.softmax(torch.randn(9, 3, generator=g).double(), -1).float()
+    pos = np.array([7, 0, 3, 5], np.int32)
+    a = oracle.predictor_loss(h, p_old, Wp, full, pos=pos)
+    b = oracle.predictor_loss(h, p_old, Wp, full[torch.from_numpy(pos).long()])
+    assert a["bad"] == 0 and abs(a["loss"] - b["loss"]) <= 1e-15
+    assert np.array_equal(a["grad"], b["grad"])
+    bad = np.array([7, 9, 3, -1], np.int32)
+    c = oracle.predictor_loss(h, p_old, Wp, full, pos=bad)
+    keep = oracle.predictor_loss(h[[0, 2]], p_old[[0, 2]], Wp, full[[7, 3]])
+    assert c["bad"] == 2 and c["kl"][1] == 0 and c["kl"][3] == 0
+    assert abs(c["loss"] * 4 - keep["loss"] * 2) <= 1e-12
+    empty = oracle.predictor_loss(h[:0], p_old[:0], Wp, full)
+    assert empty["loss"] == 0 and not np.any(empty["grad"])
+
+
+# ---- Sec. 5: top-k agreement and deviation histogram ----------------------------------------
+
+def test_route_diagnostics_match_brute_force():
+    g = torch.Generator().manual_seed(12)
+    T, N, k = 40, 9, 3
+    # probabilities on a coarse grid so that exact ties occur
+    raw = torch.randint(0, 6, (T, N), generator=g).double()
+    rho = (raw / raw.sum(1, keepdim=True).clamp(min=1)).float()
+    cached = torch.stack([torch.randperm(N, generator=g)[:k] for _ in range(T)]).int().numpy()
+    cached[3, 1] = N        # invalid
+    cached[5, 2] = cached[5, 0]  # repeated
+    r = oracle.route_diagnostics(rho, cached)
+    hist = np.zeros(k + 1, np.int64)
+    total = 0
+    rv = rho.numpy()
+    for t in range(T):
+        cur = set(sorted(range(N), key=lambda e: (-float(rv[t, e]), e))[:k])
+        seen, ov = set(), 0
+        for e in cached[t]:
+            if 0 <= e < N and e not in seen and e in cur:
+                ov += 1
+            seen.add(int(e))
+        hist[k - ov] += 1
+        total += ov
+    assert np.array_equal(r["hist"], hist) and r["overlap"] == total
+    assert r["agreement"] == total / (T * k)
+
+
+def test_route_diagnostics_identity_and_disjoint_routes():
+    g = torch.Generator().manual_seed(13)
+    T, N, k = 16, 10, 4
+    rho = torch.softmax(torch.randn(T, N, generator=g).double(), -1).float()
+    order = torch.argsort(-rho.double(), dim=1, stable=True).int().numpy()
+    same = oracle.route_diagnostics(rho, order[:, :k])
+    assert same["hist"][0] == T and same["agreement"] == 1.0
+    far = oracle.route_diagnostics(rho, order[:, -k:])
+    assert far["hist"][k] == T and far["agreement"] == 0.0
+
+
+# ---- Algorithm 2: fixed-length feature cache ------------------------------------------------
+
+@pytest.mark.parametrize("Tc", [1, 5, 37])
+def test_feature_cache_evenly_spaced_rows(Tc):
+    g = torch.Generator().manual_seed(14)
+    T, d, N = 37, 8, 6
+    h = torch.randn(T, d, generator=g).bfloat16()
+    lg = torch.randn(T, N, generator=g)
+    r = oracle.feature_cache(h, lg, Tc)
+    pos = r["pos"]
+    assert list(pos) == [c * T // Tc for c in range(Tc)] and pos[0] == 0
+    assert np.all(np.diff(pos) >= 1) and pos[-1] <= T - 1
+    assert torch.equal(r["h"], h[torch.from_numpy(pos).long()])
+    assert np.array_equal(r["p"], lg.numpy()[pos])
