@@ -54,6 +54,7 @@ typedef enum { PR2_FP32 = 0, PR2_BF16 = 1 } pr2_dtype;
 
 /* dims->flags bits */
 #define PR2_F_SYNC_STATUS 0x1u /* synchronise `stream` and turn the status word into a code */
+#define PR2_F_DELTA_LOSS 0x2u  /* pr2_predictor_loss: the delta-matching variant              */
 
 /* device status word bits (OR-ed in by the kernels; the caller zeroes the word) */
 #define PR2_STATUS_BAD_INDEX 0x1
@@ -164,6 +165,38 @@ pr2_status pr2_moe_forward_static(const pr2_dims* dims, const void* h, const int
 
 /* Size in bytes of the scratch array used by pr2_moe_forward_static (no paper counterpart). */
 size_t pr2_static_scratch_bytes(void);
+
+/*
+ * Predictive loss of one layer and its gradient w.r.t. the evolution predictor (Sec. 4.2 Eq.
+ * pr2_loss; Algorithm 3 "reconstruct the predictive distribution", "predictive KL loss").
+ * dims->T is the number T_c of cached tokens; d, N and dtype are the layer's (k is unused
+ * beyond the usual checks).
+ *  h_old [T_c, d] dtype, p_old [T_c, N] fp32: the cached route-recording features (Algorithm 2
+ *    feature cache).  W_pred [N, d] dtype: the predictor W_p.
+ *  rho [T_rho, N] fp32: the teacher, the current routing distribution Softmax(h W) of the
+ *    batch (e.g. the `probs` output of pr2_route_replay); a stop-gradient target.  Cached row c
+ *    is compared with row pos[c] (pos [T_c] int32; NULL: row c).  A pos entry outside
+ *    [0, T_rho) sets PR2_STATUS_BAD_INDEX and that row contributes nothing.
+ *  Default (Eq. pr2_loss):  z = p_old + h_old W_p^T,  rho_hat = Softmax(z),
+ *      KL_c = sum_j rho_j (log rho_j - log rho_hat_j),   dKL_c/dz = rho_hat - rho.
+ *  PR2_F_DELTA_LOSS (the appendix delta-matching variant): target q = Softmax(p - p_old),
+ *      computed as Softmax(log rho - p_old); prediction Softmax(h_old W_p^T);
+ *      KL_c = KL(q || Softmax(b)),  dKL_c/db = Softmax(b) - q.
+ *  Outputs: loss[0] = (1/T_c) sum_c KL_c (fp32, summed in double in a fixed order);
+ *    kl_tok [T_c] fp32 per-token KL_c (nullable);
+ *    grad_Wp [N, d] fp32 = (1/T_c) sum_c (dKL_c/dz)^T h_old[c] (overwritten).
+ *  T_c = 0 writes loss 0 and a zero gradient.  bf16 runs the predictor projection on tcgen05
+ *  (fp32 accumulation) and the gradient as a tcgen05 GEMM on bf16-rounded dKL/dz; fp32 runs
+ *  exact-fp32 SIMT kernels.  Deterministic.
+ *  workspace/ws_bytes: device scratch of at least pr2_predictor_loss_workspace_bytes(dims)
+ *    bytes, 256-byte aligned, not used concurrently by another call.
+ */
+size_t pr2_predictor_loss_workspace_bytes(const pr2_dims* dims);
+pr2_status pr2_predictor_loss(const pr2_dims* dims, const void* h_old, const float* p_old,
+                              const void* W_pred, const float* rho, int64_t T_rho,
+                              const int32_t* pos, float* loss, float* kl_tok, float* grad_Wp,
+                              void* workspace, size_t ws_bytes, int32_t* status_dev,
+                              void* stream);
 
 /* Static, human-readable name of a status code. */
 const char* pr2_strerror(pr2_status s);

@@ -23,6 +23,7 @@ _lib: Optional[ctypes.CDLL] = None
 PR2_OK = 0
 PR2_FP32, PR2_BF16 = 0, 1
 PR2_F_SYNC_STATUS = 0x1
+PR2_F_DELTA_LOSS = 0x2
 PR2_STATUS_BAD_INDEX = 0x1
 PR2_STATUS_TIMEOUT = 0x2
 PR2_NEAR_TIE_GAP = 1e-4
@@ -94,6 +95,11 @@ def load() -> ctypes.CDLL:
         lib.pr2_strerror.restype = ctypes.c_char_p
         lib.pr2_selftest_wait_timeout.argtypes = [P, I64, P]
         lib.pr2_selftest_wait_timeout.restype = ctypes.c_int
+        lib.pr2_predictor_loss_workspace_bytes.argtypes = [D]
+        lib.pr2_predictor_loss_workspace_bytes.restype = ctypes.c_size_t
+        lib.pr2_predictor_loss.argtypes = [D, P, P, P, P, I64, P, P, P, P, P, ctypes.c_size_t, P,
+                                           P]
+        lib.pr2_predictor_loss.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -159,12 +165,36 @@ def pr2_selftest_wait_timeout(status, timeout_ns: int, stream=None) -> int:
     return load().pr2_selftest_wait_timeout(_p(status), int(timeout_ns), _s(stream))
 
 
+def pr2_predictor_loss_workspace_bytes(dm: Dims) -> int:
+    return int(load().pr2_predictor_loss_workspace_bytes(ctypes.byref(dm)))
+
+
+def pr2_predictor_loss(dm: Dims, h_old, p_old, W_pred, rho, loss, grad, pos=None, kl_tok=None,
+                       workspace=None, ws_bytes=None, status=None, stream=None) -> int:
+    """Predictive loss (Eq. pr2_loss) and W_p gradient; ``dm.T`` = number of cached tokens and
+    ``dm.flags`` may hold PR2_F_DELTA_LOSS.  ``rho`` rows are addressed through ``pos``."""
+    if ws_bytes is None:
+        ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    T_rho = int(rho.shape[0]) if rho is not None else 0
+    return load().pr2_predictor_loss(ctypes.byref(dm), _p(h_old), _p(p_old), _p(W_pred), _p(rho),
+                                     T_rho, _p(pos), _p(loss), _p(kl_tok), _p(grad),
+                                     _p(workspace), ctypes.c_size_t(ws_bytes), _p(status),
+                                     _s(stream))
+
+
 # ---- allocation helpers (plain torch.empty on the caller's device) ---------------------------
 
 def alloc_workspace(dm: Dims, device="cuda") -> torch.Tensor:
     n = pr2_moe_workspace_bytes(dm)
     if n == 0:
         raise Pr2Error(1, "pr2_moe_workspace_bytes")
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+def alloc_loss_workspace(dm: Dims, device="cuda") -> torch.Tensor:
+    n = pr2_predictor_loss_workspace_bytes(dm)
+    if n == 0:
+        raise Pr2Error(1, "pr2_predictor_loss_workspace_bytes")
     return torch.empty(n, dtype=torch.uint8, device=device)
 
 

@@ -159,7 +159,8 @@ pr2_status route_common(const pr2_dims* dims, bool predict, const void* h, const
     if (dm.T > (int64_t{1} << 30)) return PR2_ERR_UNSUPPORTED;
     const int num_sms = num_sms_of_current_device();
     if (num_sms <= 0) return PR2_ERR_CUDA;
-    const int split = route_split(static_cast<int>(dm.T), dm.N, dm.d, predict, num_sms);
+    const int mode = predict ? kModePredict : kModeReplay;
+    const int split = route_split(static_cast<int>(dm.T), dm.N, dm.d, mode, num_sms);
     CUtensorMap tm_h, tm_w, tm_wp;
     if (!make_tmap_bf16(&tm_h, h, dm.d, dm.T, 64, kTileM) ||
         !make_tmap_bf16(&tm_w, W, dm.d, dm.N, 64, dm.N))
@@ -169,11 +170,53 @@ pr2_status route_common(const pr2_dims* dims, bool predict, const void* h, const
     } else {
       tm_wp = tm_w;
     }
-    RouteTcArgs a{static_cast<int>(dm.T), dm.d, dm.N, dm.k, idx_in, idx_out,
-                  gates, aux, near_tie, status_dev};
-    err = launch_route_tc(predict, tm_h, tm_w, tm_wp, a, split, st);
+    RouteTcArgs a{};
+    a.T = static_cast<int>(dm.T);
+    a.d = dm.d;
+    a.N = dm.N;
+    a.k = dm.k;
+    a.idx_in = idx_in;
+    a.idx_out = idx_out;
+    a.gates = gates;
+    a.logits_or_probs = aux;
+    a.near_tie = near_tie;
+    a.status = status_dev;
+    err = launch_route_tc(mode, tm_h, tm_w, tm_wp, a, split, st);
   }
   return finish(err, dm.flags, status_dev, st);
+}
+
+// ---- workspace of pr2_predictor_loss ---------------------------------------------------------
+struct LossWorkspace {
+  int32_t* status;
+  uint16_t* gt;     // bf16: [N, Tpad] dKL/dz transposed
+  float* G;         // fp32: [Tc, N] dKL/dz
+  float* kl;        // [Tpad] per-token KL when the caller passes none
+  float* partial;   // bf16: [kLossMaxSplit, N, d]
+  int Tpad;
+  size_t total;
+};
+
+LossWorkspace carve_loss(const pr2_dims& dm, uint8_t* base) {
+  LossWorkspace w{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) -> uint8_t* {
+    uint8_t* p = base ? base + off : nullptr;
+    off += (bytes + 255) & ~size_t{255};
+    return p;
+  };
+  w.Tpad = static_cast<int>((dm.T + kTileM - 1) / kTileM) * kTileM;
+  w.status = reinterpret_cast<int32_t*>(take(sizeof(int32_t)));
+  w.kl = reinterpret_cast<float*>(take(sizeof(float) * (size_t)(w.Tpad > 0 ? w.Tpad : 1)));
+  if (dm.dtype == PR2_BF16) {
+    w.gt = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * (size_t)dm.N * w.Tpad));
+    w.partial = reinterpret_cast<float*>(
+        take(sizeof(float) * (size_t)kLossMaxSplit * dm.N * (size_t)dm.d));
+  } else {
+    w.G = reinterpret_cast<float*>(take(sizeof(float) * (size_t)dm.T * dm.N));
+  }
+  w.total = off;
+  return w;
 }
 
 }  // namespace
@@ -195,6 +238,88 @@ pr2_status pr2_route_replay(const pr2_dims* dims, const void* h, const void* W_r
                             void* stream) {
   return route_common(dims, false, h, W_router, nullptr, idx, nullptr, gates, probs, nullptr,
                       status_dev, stream);
+}
+
+size_t pr2_predictor_loss_workspace_bytes(const pr2_dims* dims) {
+  if (check_dims(dims) != PR2_OK) return 0;
+  return carve_loss(*dims, nullptr).total;
+}
+
+pr2_status pr2_predictor_loss(const pr2_dims* dims, const void* h_old, const float* p_old,
+                              const void* W_pred, const float* rho, int64_t T_rho,
+                              const int32_t* pos, float* loss, float* kl_tok, float* grad_Wp,
+                              void* workspace, size_t ws_bytes, int32_t* status_dev,
+                              void* stream) {
+  pr2_status s = check_dims(dims);
+  if (s != PR2_OK) return s;
+  const pr2_dims& dm = *dims;
+  if (dm.T > (int64_t{1} << 30) - kTileM) return PR2_ERR_UNSUPPORTED;
+  if (loss == nullptr || grad_Wp == nullptr || W_pred == nullptr) return PR2_ERR_INVALID_ARG;
+  if (dm.T > 0 && (h_old == nullptr || p_old == nullptr || rho == nullptr || T_rho < 1))
+    return PR2_ERR_INVALID_ARG;
+  if ((dm.flags & PR2_F_SYNC_STATUS) && status_dev == nullptr) return PR2_ERR_INVALID_ARG;
+  const void* al[] = {h_old, p_old, W_pred, rho, loss, kl_tok, grad_Wp};
+  for (const void* p : al)
+    if (p != nullptr && !aligned16(p)) return PR2_ERR_INVALID_ARG;
+  const LossWorkspace probe = carve_loss(dm, nullptr);
+  if (workspace == nullptr || ws_bytes < probe.total ||
+      (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+    return PR2_ERR_WORKSPACE;
+  const LossWorkspace w = carve_loss(dm, static_cast<uint8_t*>(workspace));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int32_t* status = status_dev ? status_dev : w.status;
+  cudaError_t err = cudaSuccess;
+  if (status_dev == nullptr) err = cudaMemsetAsync(w.status, 0, sizeof(int32_t), st);
+  if (err == cudaSuccess && dm.T == 0) {  // no cached token: loss 0, gradient 0
+    err = cudaMemsetAsync(loss, 0, sizeof(float), st);
+    if (err == cudaSuccess)
+      err = cudaMemsetAsync(grad_Wp, 0, sizeof(float) * (size_t)dm.N * dm.d, st);
+    return finish(err, dm.flags, status_dev, st);
+  }
+  if (err != cudaSuccess) return PR2_ERR_CUDA;
+  const int Tc = static_cast<int>(dm.T);
+  float* kl = kl_tok ? kl_tok : w.kl;
+  const int delta = (dm.flags & PR2_F_DELTA_LOSS) ? 1 : 0;
+  GradArgs g{dm.N, dm.d, Tc, w.Tpad, 1, nullptr, grad_Wp, kl, loss, status};
+  if (dm.dtype == PR2_FP32) {
+    err = launch_loss_simt(static_cast<const float*>(h_old), p_old,
+                           static_cast<const float*>(W_pred), rho, T_rho, pos, delta, Tc, dm.d,
+                           dm.N, kl, w.G, status, st);
+    if (err == cudaSuccess)
+      err = launch_loss_grad_simt(w.G, static_cast<const float*>(h_old), Tc, dm.d, dm.N,
+                                  grad_Wp, st);
+    if (err == cudaSuccess) err = launch_loss_finish(g, st);
+    return finish(err, dm.flags, status_dev, st);
+  }
+  const int num_sms = num_sms_of_current_device();
+  if (num_sms <= 0) return PR2_ERR_CUDA;
+  CUtensorMap tm_h, tm_w, tm_gt, tm_hmn;
+  if (!make_tmap_bf16(&tm_h, h_old, dm.d, dm.T, 64, kTileM) ||
+      !make_tmap_bf16(&tm_w, W_pred, dm.d, dm.N, 64, dm.N) ||
+      !make_tmap_bf16(&tm_gt, w.gt, w.Tpad, dm.N, 64, kTileM) ||
+      !make_tmap_bf16(&tm_hmn, h_old, dm.d, dm.T, 64, 64))
+    return PR2_ERR_CUDA;
+  RouteTcArgs a{};
+  a.T = Tc;
+  a.d = dm.d;
+  a.N = dm.N;
+  a.k = dm.k;
+  a.status = status;
+  a.p_old = p_old;
+  a.rho = rho;
+  a.pos = pos;
+  a.T_rho = T_rho;
+  a.delta = delta;
+  a.kl_tok = kl;
+  a.gt = w.gt;
+  a.Tpad = w.Tpad;
+  const int split = route_split(Tc, dm.N, dm.d, kModeLoss, num_sms);
+  err = launch_route_tc(kModeLoss, tm_h, tm_w, tm_w, a, split, st);
+  g.split = loss_grad_split(dm.N, dm.d, w.Tpad, num_sms);
+  g.partial = w.partial;
+  if (err == cudaSuccess) err = launch_loss_grad_tc(tm_gt, tm_hmn, g, st);
+  if (err == cudaSuccess) err = launch_loss_finish(g, st);
+  return finish(err, dm.flags, status_dev, st);
 }
 
 size_t pr2_moe_workspace_bytes(const pr2_dims* dims) {

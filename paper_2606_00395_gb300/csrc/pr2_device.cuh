@@ -175,6 +175,21 @@ __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t smem_addr) {
   return desc;
 }
 
+// Descriptor of an MN-major operand tile with the 128-byte swizzle: each 128-B row holds 64
+// consecutive MN elements of one K index, 8 consecutive K rows form one 1024-B swizzle atom
+// (stride byte offset 1024 between 8-row K groups), and further 64-element MN chunks follow
+// `mn_chunk_bytes` apart (leading byte offset).  A K step of 16 advances the start by 2048 B.
+__device__ __forceinline__ uint64_t umma_desc_sw128_mn(uint32_t smem_addr,
+                                                       uint32_t mn_chunk_bytes) {
+  uint64_t desc = 0;
+  desc |= static_cast<uint64_t>((smem_addr & 0x3FFFFu) >> 4);
+  desc |= static_cast<uint64_t>((mn_chunk_bytes >> 4) & 0x3FFFu) << 16;
+  desc |= static_cast<uint64_t>(1024u >> 4) << 32;
+  desc |= static_cast<uint64_t>(1u) << 46;
+  desc |= static_cast<uint64_t>(2u) << 61;
+  return desc;
+}
+
 // Instruction descriptor of tcgen05.mma kind::f16: D fp32, A and B bf16, both K-major, M x N.
 __host__ __device__ constexpr uint32_t umma_idesc_bf16(int M, int N) {
   return (1u << 4)                                   // D format: f32
@@ -182,6 +197,10 @@ __host__ __device__ constexpr uint32_t umma_idesc_bf16(int M, int N) {
          | (1u << 10)                                // B format: bf16
          | (static_cast<uint32_t>(N >> 3) << 17)     // N / 8
          | (static_cast<uint32_t>(M >> 4) << 24);    // M / 16
+}
+// Same with B given MN-major (bit 16).
+__host__ __device__ constexpr uint32_t umma_idesc_bf16_bmn(int M, int N) {
+  return umma_idesc_bf16(M, N) | (1u << 16);
 }
 
 // D[tmem] (+)= A[smem] x B[smem]^T, one instruction issued by a single thread.

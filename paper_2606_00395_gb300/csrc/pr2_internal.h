@@ -56,6 +56,13 @@ cudaError_t launch_route_simt(const pr2_dims& dm, bool predict, const float* h, 
                               float* gates, float* logits_or_probs, int64_t* near_tie,
                               int32_t* status, cudaStream_t st);
 
+// Modes of the tensor-core routing kernel (route_tc.cu).
+enum RouteMode : int {
+  kModeReplay = 0,   // rho = Softmax(h W^T), gates = rho[idx_in]
+  kModePredict = 1,  // z = h W^T + h W_p^T, top-k, gates = rho_hat[idx]
+  kModeLoss = 2,     // predictive loss: z = p_old + h_old W_p^T against a teacher rho
+};
+
 struct RouteTcArgs {
   int T, d, N, k;
   const int32_t* idx_in;   // replay: cached route
@@ -64,10 +71,19 @@ struct RouteTcArgs {
   float* logits_or_probs;  // predict: p_old [T,N]; replay: rho [T,N]; nullable
   int64_t* near_tie;
   int32_t* status;
+  // kModeLoss only (h = h_old, W = W_p)
+  const float* p_old;      // [T, N] cached router logits
+  const float* rho;        // [T_rho, N] teacher probabilities
+  const int32_t* pos;      // [T] teacher row of each cached row (nullable: row t)
+  int64_t T_rho;
+  int delta;               // 1: delta-matching variant
+  float* kl_tok;           // [T] per-token KL
+  uint16_t* gt;            // [N, Tpad] bf16 bits of dKL/dz, transposed; rows t >= T hold 0
+  int Tpad;                // multiple of 128, >= T
 };
 // CTAs of the cluster that splits K for one 128-token tile (1 = no split).
-int route_split(int T, int N, int d, bool predict, int num_sms);
-cudaError_t launch_route_tc(bool predict, const CUtensorMap& tm_h, const CUtensorMap& tm_w,
+int route_split(int T, int N, int d, int mode, int num_sms);
+cudaError_t launch_route_tc(int mode, const CUtensorMap& tm_h, const CUtensorMap& tm_w,
                             const CUtensorMap& tm_wp, const RouteTcArgs& a, int split,
                             cudaStream_t st);
 
@@ -119,6 +135,31 @@ cudaError_t launch_expert_tc(bool swiglu, const CUtensorMap& tm_a, const CUtenso
                              cudaStream_t st);
 cudaError_t launch_expert_simt(bool swiglu, const float* A, const float* Wb0, const float* Wb1,
                                const GemmArgs& g, cudaStream_t st);
+
+// ---- predictive loss gradient (predictor.cu) ---------------------------------------------
+// grad_Wp = (1/T_c) G^T h_old with G = dKL/dz.  bf16: split-K tcgen05 GEMM over tokens into
+// `partial` [split, N, d] fp32, then a fixed-order reduction.  fp32: SIMT kernels.
+struct GradArgs {
+  int N, d, Tc, Tpad;
+  int split;              // token-block split of the GEMM
+  float* partial;         // [split, N, d]
+  float* grad;            // [N, d]
+  const float* kl_tok;    // [Tc]
+  float* loss;            // [1]
+  int32_t* status;
+};
+constexpr int kLossMaxSplit = 16;
+int loss_grad_split(int N, int d, int Tpad, int num_sms);
+cudaError_t launch_loss_grad_tc(const CUtensorMap& tm_gt, const CUtensorMap& tm_h,
+                                const GradArgs& g, cudaStream_t st);
+cudaError_t launch_loss_finish(const GradArgs& g, cudaStream_t st);
+// fp32 path: per-token KL and G [Tc, N] (row-major), then the gradient.
+cudaError_t launch_loss_simt(const float* h_old, const float* p_old, const float* Wp,
+                             const float* rho, int64_t T_rho, const int32_t* pos, int delta,
+                             int Tc, int d, int N, float* kl_tok, float* G, int32_t* status,
+                             cudaStream_t st);
+cudaError_t launch_loss_grad_simt(const float* G, const float* h_old, int Tc, int d, int N,
+                                  float* grad, cudaStream_t st);
 
 // ---- self test (api.cu) --------------------------------------------------------------------
 cudaError_t launch_wait_selftest(int32_t* status, int64_t timeout_ns, cudaStream_t st);

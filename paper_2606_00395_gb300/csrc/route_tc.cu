@@ -148,11 +148,13 @@ __device__ __forceinline__ bool predict_write(const uint64_t (&key)[16], float m
   return (a.k < a.N) && (pk - pk1 < (float)PR2_NEAR_TIE_GAP);
 }
 
-template <bool predict, int split>
+template <int kMode, int split>
 __global__ void __launch_bounds__(kThreads, 1)
     route_tc_kernel(const __grid_constant__ CUtensorMap tm_h,
                     const __grid_constant__ CUtensorMap tm_w,
                     const __grid_constant__ CUtensorMap tm_wp, RouteTcArgs a) {
+  constexpr bool predict = kMode == kModePredict;
+  constexpr bool loss = kMode == kModeLoss;
   extern __shared__ __align__(16) uint8_t smem_raw[];
   const int N = a.N, k = a.k;
   const RouteSmemLayout L = route_layout(N, predict);
@@ -285,7 +287,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // replay: cached indices, validated (range, duplicates) while the K blocks run
   int e_s[kMaxTopK];
   bool bad = false;
-  if (!predict) {
+  if (kMode == kModeReplay) {
 #pragma unroll
     for (int s = 0; s < kMaxTopK; ++s) {
       int e = -1;
@@ -366,7 +368,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // One pass over this thread's experts, 16 at a time: running max m and sum of exp(z - m),
   // (predict) the top-16 keys, (replay) the z of the cached slots.
-  if (epi) {
+  if (epi && !loss) {
     bool tie = false;
     float m = -FLT_MAX, sum = 0.f;
     uint64_t top[16];
@@ -440,7 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         merge16_desc(top, other);
       }
       if (have && live && part == 0) tie = predict_write(top, mx, inv_s, t, a);
-    } else {
+    } else if (!loss) {
       // Each valid slot's z is held by the one thread owning its expert; the others hold 0.
 #pragma unroll
       for (int s = 0; s < kMaxTopK; ++s)
@@ -476,6 +478,119 @@ __global__ void __launch_bounds__(kThreads, 1)
                 static_cast<unsigned long long>(__popc(ties)));
     tc_fence_before();
   }
+  if (epi && loss) {
+    // Predictive loss (Eq. pr2_loss, Algorithm 3) of cached row t over experts [fe0, fe0+nr):
+    //   standard: prediction Softmax(v), v = p_old + b;  target rho (row pos[t] of the teacher)
+    //   delta:    prediction Softmax(b);  target Softmax(u), u = log rho - p_old
+    // KL_t = sum_j tgt_j (log tgt_j - log pred_j);  dKL_t/dv_j = pred_j - tgt_j, stored bf16
+    // and transposed for the gradient GEMM.  Two passes: normalisers, then terms.
+    const bool delta = a.delta != 0;
+    int64_t r = 0;
+    bool okp = false;
+    if (live) {
+      r = a.pos != nullptr ? static_cast<int64_t>(a.pos[t]) : t;
+      okp = r >= 0 && r < a.T_rho;
+      if (!okp && part == 0 && a.status != nullptr) atomicOr(a.status, PR2_STATUS_BAD_INDEX);
+    }
+    const bool use = have && okp;
+    const float* po = a.p_old + (live ? t : 0) * N;
+    const float* tr = a.rho + (okp ? r : 0) * N;
+    auto row16 = [&](const float* src, int c, float (&v)[16]) {
+      const float4* q = reinterpret_cast<const float4*>(src + c);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float4 x = q[j];
+        v[4 * j] = x.x;
+        v[4 * j + 1] = x.y;
+        v[4 * j + 2] = x.z;
+        v[4 * j + 3] = x.w;
+      }
+    };
+    float m1 = -FLT_MAX, s1 = 0.f, m2 = -FLT_MAX, s2 = 0.f;
+    for (int c0 = fe0; c0 < fe0 + nr; c0 += 16) {
+      uint32_t rb[16];
+      load16(c0, rb);
+      if (use) {
+        float pv[16], rv[16], v[16], u[16];
+        row16(po, c0, pv);
+        row16(tr, c0, rv);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const float b = __uint_as_float(rb[j]);
+          v[j] = delta ? b : pv[j] + b;
+          u[j] = rv[j] > 0.f ? logf(rv[j]) - pv[j] : -INFINITY;
+        }
+        float cm = v[0];
+#pragma unroll
+        for (int j = 1; j < 16; ++j) cm = fmaxf(cm, v[j]);
+        float nm = fmaxf(m1, cm), cs = 0.f;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) cs += expf(v[j] - nm);
+        s1 = s1 * expf(m1 - nm) + cs;
+        m1 = nm;
+        if (delta) {
+          cm = u[0];
+#pragma unroll
+          for (int j = 1; j < 16; ++j) cm = fmaxf(cm, u[j]);
+          nm = fmaxf(m2, cm);
+          cs = 0.f;
+#pragma unroll
+          for (int j = 0; j < 16; ++j) cs += expf(u[j] - nm);
+          s2 = s2 * expf(m2 - nm) + cs;
+          m2 = nm;
+        }
+      }
+    }
+    float mx1 = m1, mx2 = m2;
+#pragma unroll
+    for (int o = 1; o < split; o <<= 1) {
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+      mx2 = fmaxf(mx2, __shfl_xor_sync(0xffffffffu, mx2, o));
+    }
+    float f1 = s1 * expf(m1 - mx1), f2 = s2 * expf(m2 - mx2);
+#pragma unroll
+    for (int o = 1; o < split; o <<= 1) {
+      f1 += __shfl_xor_sync(0xffffffffu, f1, o);
+      f2 += __shfl_xor_sync(0xffffffffu, f2, o);
+    }
+    const float l1 = mx1 + logf(f1), l2 = mx2 + logf(f2);  // log normalisers
+    float kl = 0.f;
+    for (int c0 = fe0; c0 < fe0 + nr; c0 += 16) {
+      uint32_t rb[16];
+      load16(c0, rb);
+      float g[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) g[j] = 0.f;
+      if (use) {
+        float pv[16], rv[16];
+        row16(po, c0, pv);
+        row16(tr, c0, rv);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const float b = __uint_as_float(rb[j]);
+          const float lp = (delta ? b : pv[j] + b) - l1;  // log prediction
+          float tg, lt;
+          if (delta) {
+            lt = rv[j] > 0.f ? logf(rv[j]) - pv[j] - l2 : -INFINITY;
+            tg = rv[j] > 0.f ? expf(lt) : 0.f;
+          } else {
+            tg = rv[j];
+            lt = rv[j] > 0.f ? logf(rv[j]) : 0.f;
+          }
+          if (tg > 0.f) kl += tg * (lt - lp);
+          g[j] = expf(lp) - tg;
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 16; ++j)
+        a.gt[static_cast<int64_t>(c0 + j) * a.Tpad + t] =
+            __bfloat16_as_ushort(__float2bfloat16_rn(g[j]));
+    }
+#pragma unroll
+    for (int o = 1; o < split; o <<= 1) kl += __shfl_xor_sync(0xffffffffu, kl, o);
+    if (live && part == 0) a.kl_tok[t] = use ? kl : 0.f;
+    tc_fence_before();
+  }
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
@@ -483,20 +598,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <bool kPredict, int kSplit>
+template <int kMode, int kSplit>
 cudaError_t set_smem_attr(int N) {
-  return cudaFuncSetAttribute(route_tc_kernel<kPredict, kSplit>,
+  return cudaFuncSetAttribute(route_tc_kernel<kMode, kSplit>,
                               cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              route_layout(N, kPredict).total);
+                              route_layout(N, kMode == kModePredict).total);
 }
 
-template <bool kPredict, int kSplit>
+template <int kMode, int kSplit>
 cudaError_t launch_split(const CUtensorMap& tm_h, const CUtensorMap& tm_w,
                          const CUtensorMap& tm_wp, const RouteTcArgs& a, int tiles,
                          cudaStream_t st, int* max_clusters) {
-  cudaError_t err = set_smem_attr<kPredict, kSplit>(a.N);
+  cudaError_t err = set_smem_attr<kMode, kSplit>(a.N);
   if (err != cudaSuccess) return err;
-  const size_t smem = route_layout(a.N, kPredict).total;
+  const size_t smem = route_layout(a.N, kMode == kModePredict).total;
   if (max_clusters != nullptr) {  // occupancy query only
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(tiles * kSplit);
@@ -509,30 +624,44 @@ cudaError_t launch_split(const CUtensorMap& tm_h, const CUtensorMap& tm_w,
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaOccupancyMaxActiveClusters(max_clusters, route_tc_kernel<kPredict, kSplit>, &cfg);
+    return cudaOccupancyMaxActiveClusters(max_clusters, route_tc_kernel<kMode, kSplit>, &cfg);
   }
-  return launch_pdl(route_tc_kernel<kPredict, kSplit>, dim3(tiles * kSplit), dim3(kThreads), smem,
+  return launch_pdl(route_tc_kernel<kMode, kSplit>, dim3(tiles * kSplit), dim3(kThreads), smem,
                     st, kSplit, tm_h, tm_w, tm_wp, a);
 }
 
-template <bool kPredict>
-cudaError_t launch_any(const CUtensorMap& tm_h, const CUtensorMap& tm_w, const CUtensorMap& tm_wp,
-                       const RouteTcArgs& a, int split, int tiles, cudaStream_t st,
-                       int* max_clusters) {
+template <int kMode>
+cudaError_t launch_splits(const CUtensorMap& tm_h, const CUtensorMap& tm_w,
+                          const CUtensorMap& tm_wp, const RouteTcArgs& a, int split, int tiles,
+                          cudaStream_t st, int* max_clusters) {
   switch (split) {
-    case 1: return launch_split<kPredict, 1>(tm_h, tm_w, tm_wp, a, tiles, st, max_clusters);
-    case 2: return launch_split<kPredict, 2>(tm_h, tm_w, tm_wp, a, tiles, st, max_clusters);
-    case 4: return launch_split<kPredict, 4>(tm_h, tm_w, tm_wp, a, tiles, st, max_clusters);
-    case 8: return launch_split<kPredict, 8>(tm_h, tm_w, tm_wp, a, tiles, st, max_clusters);
+    case 1: return launch_split<kMode, 1>(tm_h, tm_w, tm_wp, a, tiles, st, max_clusters);
+    case 2: return launch_split<kMode, 2>(tm_h, tm_w, tm_wp, a, tiles, st, max_clusters);
+    case 4: return launch_split<kMode, 4>(tm_h, tm_w, tm_wp, a, tiles, st, max_clusters);
+    case 8: return launch_split<kMode, 8>(tm_h, tm_w, tm_wp, a, tiles, st, max_clusters);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_any(int mode, const CUtensorMap& tm_h, const CUtensorMap& tm_w,
+                       const CUtensorMap& tm_wp, const RouteTcArgs& a, int split, int tiles,
+                       cudaStream_t st, int* max_clusters) {
+  switch (mode) {
+    case kModeReplay:
+      return launch_splits<kModeReplay>(tm_h, tm_w, tm_wp, a, split, tiles, st, max_clusters);
+    case kModePredict:
+      return launch_splits<kModePredict>(tm_h, tm_w, tm_wp, a, split, tiles, st, max_clusters);
+    case kModeLoss:
+      return launch_splits<kModeLoss>(tm_h, tm_w, tm_wp, a, split, tiles, st, max_clusters);
     default: return cudaErrorInvalidValue;
   }
 }
 
 // Clusters of `split` CTAs of this kernel that can be resident at once (0 on error), cached
 // per device and shape.
-int max_active_clusters(bool predict, int split, int N) {
+int max_active_clusters(int mode, int split, int N) {
   struct Entry {
-    int dev, predict, split, N, clusters;
+    int dev, mode, split, N, clusters;
   };
   static std::mutex mu;
   static Entry cache[64];
@@ -541,40 +670,38 @@ int max_active_clusters(bool predict, int split, int N) {
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
   std::lock_guard<std::mutex> lock(mu);
   for (int i = 0; i < used; ++i)
-    if (cache[i].dev == dev && cache[i].predict == (predict ? 1 : 0) &&
-        cache[i].split == split && cache[i].N == N)
+    if (cache[i].dev == dev && cache[i].mode == mode && cache[i].split == split &&
+        cache[i].N == N)
       return cache[i].clusters;
   RouteTcArgs probe{};
   probe.N = N;
   CUtensorMap none{};
   int clusters = 0;
-  const cudaError_t err =
-      predict ? launch_any<true>(none, none, none, probe, split, 1, nullptr, &clusters)
-              : launch_any<false>(none, none, none, probe, split, 1, nullptr, &clusters);
+  const cudaError_t err = launch_any(mode, none, none, none, probe, split, 1, nullptr, &clusters);
   if (err != cudaSuccess) {
     (void)cudaGetLastError();
     clusters = 0;
   }
-  if (used < 64) cache[used++] = Entry{dev, predict ? 1 : 0, split, N, clusters};
+  if (used < 64) cache[used++] = Entry{dev, mode, split, N, clusters};
   return clusters;
 }
 
 }  // namespace
 
-int route_split(int T, int N, int d, bool predict, int num_sms) {
-  const RouteSmemLayout L = route_layout(N, predict);
+int route_split(int T, int N, int d, int mode, int num_sms) {
+  const RouteSmemLayout L = route_layout(N, mode == kModePredict);
   const int tiles = (T + kTileM - 1) / kTileM;
   const int KB = d / kBK;
   if (route_recv_bytes(L.b_rows) > L.stages * L.stage_bytes) return 1;
   for (int s = kMaxSplit; s > 1; s >>= 1) {
     if (N % s != 0 || (N / s) % 16 != 0 || KB % s != 0 || tiles * s > num_sms) continue;
-    if (max_active_clusters(predict, s, N) < tiles) continue;  // must fit in one wave
+    if (max_active_clusters(mode, s, N) < tiles) continue;  // must fit in one wave
     return s;
   }
   return 1;
 }
 
-cudaError_t launch_route_tc(bool predict, const CUtensorMap& tm_h, const CUtensorMap& tm_w,
+cudaError_t launch_route_tc(int mode, const CUtensorMap& tm_h, const CUtensorMap& tm_w,
                             const CUtensorMap& tm_wp, const RouteTcArgs& a, int split,
                             cudaStream_t st) {
   if (a.T == 0) return cudaSuccess;
@@ -582,8 +709,7 @@ cudaError_t launch_route_tc(bool predict, const CUtensorMap& tm_h, const CUtenso
       (a.d / kBK) % split != 0)
     return cudaErrorInvalidValue;
   const int tiles = (a.T + kTileM - 1) / kTileM;
-  return predict ? launch_any<true>(tm_h, tm_w, tm_wp, a, split, tiles, st, nullptr)
-                 : launch_any<false>(tm_h, tm_w, tm_wp, a, split, tiles, st, nullptr);
+  return launch_any(mode, tm_h, tm_w, tm_wp, a, split, tiles, st, nullptr);
 }
 
 }  // namespace pr2

@@ -108,3 +108,39 @@ def test_selftest_rejects_out_of_range_limits(lib):
     assert lib.pr2_selftest_wait_timeout(None, 1000, None) == 1
     assert lib.pr2_selftest_wait_timeout(ctypes.c_void_p(256), 10, None) == 1
     assert lib.pr2_selftest_wait_timeout(ctypes.c_void_p(256), 10 ** 10, None) == 1
+
+
+def test_predictor_loss_rejects_bad_arguments_on_the_host(lib):
+    dm = B.dims(256, 2048, 128, 8, 768)
+    fake = ctypes.c_void_p(256)
+    ws = B.pr2_predictor_loss_workspace_bytes(dm)
+    assert ws > 0
+    # bf16 workspace holds dKL/dz (N x T_c) and the split-K gradient partials
+    assert ws >= 128 * 256 * 2 + 16 * 128 * 2048 * 4
+    ok = [ctypes.byref(dm), fake, fake, fake, fake, ctypes.c_int64(256), None, fake, None, fake]
+    # missing output / input pointers
+    bad_loss = list(ok)
+    bad_loss[7] = None
+    assert lib.pr2_predictor_loss(*bad_loss, fake, ctypes.c_size_t(ws), None, None) == 1
+    bad_h = list(ok)
+    bad_h[1] = None
+    assert lib.pr2_predictor_loss(*bad_h, fake, ctypes.c_size_t(ws), None, None) == 1
+    no_teacher = list(ok)
+    no_teacher[5] = ctypes.c_int64(0)
+    assert lib.pr2_predictor_loss(*no_teacher, fake, ctypes.c_size_t(ws), None, None) == 1
+    odd = list(ok)
+    odd[2] = ctypes.c_void_p(260)
+    assert lib.pr2_predictor_loss(*odd, fake, ctypes.c_size_t(ws), None, None) == 1
+    # workspace too small, missing or misaligned
+    assert lib.pr2_predictor_loss(*ok, fake, ctypes.c_size_t(ws - 1), None, None) == 6
+    assert lib.pr2_predictor_loss(*ok, None, ctypes.c_size_t(ws), None, None) == 6
+    assert lib.pr2_predictor_loss(*ok, ctypes.c_void_p(512 + 16), ctypes.c_size_t(ws), None,
+                                  None) == 6
+    # unsupported layer shape
+    dmu = B.dims(256, 2000, 128, 8, 768)
+    assert lib.pr2_predictor_loss(ctypes.byref(dmu), *ok[1:], fake, ctypes.c_size_t(ws), None,
+                                  None) == 2
+    # sync-status needs a status word
+    dms = B.dims(256, 2048, 128, 8, 768, flags=B.PR2_F_SYNC_STATUS | B.PR2_F_DELTA_LOSS)
+    assert lib.pr2_predictor_loss(ctypes.byref(dms), *ok[1:], fake, ctypes.c_size_t(1 << 40),
+                                  None, None) == 1
