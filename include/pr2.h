@@ -198,6 +198,34 @@ pr2_status pr2_predictor_loss(const pr2_dims* dims, const void* h_old, const flo
                               void* workspace, size_t ws_bytes, int32_t* status_dev,
                               void* stream);
 
+/*
+ * Route tracking of a cached route against the current router (Sec. 5 "Top-k Agreement and
+ * Route KL", "Deviation Tails").  For each of the dims->T tokens: I_t = TopK(rho_t, k) of the
+ * current routing distribution rho [T, N] fp32 (e.g. the probs output of pr2_route_replay;
+ * ties to the lower expert as in Eq. pr2_route), Î_t = idx_cached[t] ([T, k] int32, the
+ * replayed route); overlap_t = |Î_t ∩ I_t|, where a cached entry outside [0, N) or repeated in
+ * its token never matches.  ACCUMULATES hist[k - overlap_t] += 1 (int64 [k+1], the deviation
+ * count of "Deviation Tails") and overlap_sum[0] += overlap_t; the caller zeroes both, so that
+ * layers can be summed.  Top-k agreement = overlap_sum / (T k).  Exact (integer atomics).
+ * Needs k <= 32.  The route KL of Sec. 5 is the loss value of pr2_predictor_loss.
+ */
+pr2_status pr2_route_diagnostics(const pr2_dims* dims, const float* rho,
+                                 const int32_t* idx_cached, int64_t* hist, int64_t* overlap_sum,
+                                 void* stream);
+
+/*
+ * Fixed-length feature-cache writer (Algorithm 2: store the route-recording features
+ * (h_old, p_old) of the retained positions; App.: T_c positions drawn by uniform sub-sampling
+ * along the rollout).  The T_c <= dims->T retained positions are evenly spaced,
+ * pos[c] = floor(c T / T_c) (int32 [T_c]; T_c = T keeps every token), and
+ * cache_h[c] = h[pos[c]] ([T_c, d], dims->dtype, bits copied), cache_p[c] = logits_old[pos[c]]
+ * ([T_c, N] fp32; both NULL to skip).  logits_old is the p_old output of pr2_route_predict.
+ * Cache size T_c (2 d + 4 N) bytes per layer for bf16 h (Table 4).
+ */
+pr2_status pr2_feature_cache_write(const pr2_dims* dims, int64_t T_c, const void* h,
+                                   const float* logits_old, int32_t* pos, void* cache_h,
+                                   float* cache_p, void* stream);
+
 /* Static, human-readable name of a status code. */
 const char* pr2_strerror(pr2_status s);
 

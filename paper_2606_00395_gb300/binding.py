@@ -100,6 +100,10 @@ def load() -> ctypes.CDLL:
         lib.pr2_predictor_loss.argtypes = [D, P, P, P, P, I64, P, P, P, P, P, ctypes.c_size_t, P,
                                            P]
         lib.pr2_predictor_loss.restype = ctypes.c_int
+        lib.pr2_route_diagnostics.argtypes = [D, P, P, P, P, P]
+        lib.pr2_route_diagnostics.restype = ctypes.c_int
+        lib.pr2_feature_cache_write.argtypes = [D, I64, P, P, P, P, P, P]
+        lib.pr2_feature_cache_write.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -180,6 +184,18 @@ def pr2_predictor_loss(dm: Dims, h_old, p_old, W_pred, rho, loss, grad, pos=None
                                      T_rho, _p(pos), _p(loss), _p(kl_tok), _p(grad),
                                      _p(workspace), ctypes.c_size_t(ws_bytes), _p(status),
                                      _s(stream))
+
+
+def pr2_route_diagnostics(dm: Dims, rho, idx_cached, hist, overlap_sum, stream=None) -> int:
+    """Accumulate the deviation histogram (int64 [k+1]) and the overlap sum (int64 [1])."""
+    return load().pr2_route_diagnostics(ctypes.byref(dm), _p(rho), _p(idx_cached), _p(hist),
+                                        _p(overlap_sum), _s(stream))
+
+
+def pr2_feature_cache_write(dm: Dims, Tc: int, h, logits_old, pos, cache_h, cache_p,
+                            stream=None) -> int:
+    return load().pr2_feature_cache_write(ctypes.byref(dm), int(Tc), _p(h), _p(logits_old),
+                                          _p(pos), _p(cache_h), _p(cache_p), _s(stream))
 
 
 # ---- allocation helpers (plain torch.empty on the caller's device) ---------------------------

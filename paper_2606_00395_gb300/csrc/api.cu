@@ -322,6 +322,41 @@ pr2_status pr2_predictor_loss(const pr2_dims* dims, const void* h_old, const flo
   return finish(err, dm.flags, status_dev, st);
 }
 
+pr2_status pr2_route_diagnostics(const pr2_dims* dims, const float* rho, const int32_t* idx_cached,
+                                 int64_t* hist, int64_t* overlap_sum, void* stream) {
+  pr2_status s = check_dims(dims);
+  if (s != PR2_OK) return s;
+  const pr2_dims& dm = *dims;
+  if (dm.k > kMaxTopKSimt) return PR2_ERR_UNSUPPORTED;
+  if (hist == nullptr || overlap_sum == nullptr) return PR2_ERR_INVALID_ARG;
+  if (dm.T == 0) return PR2_OK;
+  if (rho == nullptr || idx_cached == nullptr || !aligned16(rho)) return PR2_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  return finish(launch_diagnostics(rho, idx_cached, dm.T, dm.N, dm.k, hist, overlap_sum, st),
+                dm.flags & ~PR2_F_SYNC_STATUS, nullptr, st);
+}
+
+pr2_status pr2_feature_cache_write(const pr2_dims* dims, int64_t T_c, const void* h,
+                                   const float* logits_old, int32_t* pos, void* cache_h,
+                                   float* cache_p, void* stream) {
+  pr2_status s = check_dims(dims);
+  if (s != PR2_OK) return s;
+  const pr2_dims& dm = *dims;
+  if (T_c < 0 || T_c > dm.T || dm.T > (int64_t{1} << 31) - 1) return PR2_ERR_INVALID_ARG;
+  if (T_c == 0) return PR2_OK;
+  if (h == nullptr || pos == nullptr || cache_h == nullptr) return PR2_ERR_INVALID_ARG;
+  if ((logits_old == nullptr) != (cache_p == nullptr)) return PR2_ERR_INVALID_ARG;
+  if (!aligned16(h) || !aligned16(cache_h)) return PR2_ERR_INVALID_ARG;
+  const int esz = static_cast<int>(esize(dm));
+  if ((static_cast<int64_t>(dm.d) * esz) % 16 != 0) return PR2_ERR_UNSUPPORTED;
+  const int num_sms = num_sms_of_current_device();
+  if (num_sms <= 0) return PR2_ERR_CUDA;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  return finish(launch_feature_cache(h, logits_old, dm.T, T_c, dm.d, dm.N, esz, pos, cache_h,
+                                     cache_p, num_sms, st),
+                dm.flags & ~PR2_F_SYNC_STATUS, nullptr, st);
+}
+
 size_t pr2_moe_workspace_bytes(const pr2_dims* dims) {
   if (check_dims(dims) != PR2_OK) return 0;
   return carve(*dims, nullptr).total;

@@ -1,0 +1,136 @@
+// Route-tracking diagnostics (Sec. 5 "Top-k Agreement and Route KL", "Deviation Tails") and the
+// fixed-length feature-cache writer (Algorithm 2, App. "uniform sub-sampling").
+//
+// Diagnostics: one warp per token.  Lane l holds rho[t, 32 j + l]; k rounds of warp argmax
+// (largest value, lower expert on equal values, as TopK of Eq. pr2_route) mark I_t = TopK(rho_t,
+// k); overlap_t = |Î_t ∩ I_t| counts the cached entries (in range, not repeated) that are
+// marked.  hist[k - overlap_t] and sum_t overlap_t are accumulated with 64-bit integer atomics
+// (order-independent, so exact and deterministic).
+// Feature cache: row c of the cache is row pos_c = floor(c T / T_c) of the batch; one warp per
+// cached row copies h (16-byte vectors) and the fp32 router logits.
+#include "pr2_device.cuh"
+#include "pr2_internal.h"
+
+namespace pr2 {
+namespace {
+
+constexpr int kPerLane = kMaxExperts / 32;
+constexpr int kWarps = 8;
+
+__global__ void __launch_bounds__(kWarps * 32)
+    diagnostics_kernel(const float* __restrict__ rho, const int32_t* __restrict__ cached,
+                       int64_t T, int N, int k, unsigned long long* __restrict__ hist,
+                       unsigned long long* __restrict__ overlap_sum) {
+  __shared__ unsigned int sh_hist[kMaxTopKSimt + 1];
+  __shared__ unsigned int sh_sum;
+  pdl_wait();
+  pdl_trigger();
+  for (int i = threadIdx.x; i <= k; i += blockDim.x) sh_hist[i] = 0u;
+  if (threadIdx.x == 0) sh_sum = 0u;
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  const int64_t t = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
+  if (t < T) {
+    const float* row = rho + t * N;
+    float v[kPerLane];
+#pragma unroll
+    for (int j = 0; j < kPerLane; ++j) {
+      const int e = j * 32 + lane;
+      v[j] = e < N ? row[e] : 0.f;
+    }
+    unsigned taken = 0u;  // bit j: expert 32 j + lane is in I_t
+    for (int r = 0; r < k; ++r) {
+      float bv = 0.f;
+      int bi = 0x7fffffff;
+#pragma unroll
+      for (int j = 0; j < kPerLane; ++j) {
+        const int e = j * 32 + lane;
+        if (e < N && !((taken >> j) & 1u) && (bi == 0x7fffffff || v[j] > bv)) {
+          bv = v[j];
+          bi = e;
+        }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+        if (oi != 0x7fffffff && (bi == 0x7fffffff || ov > bv || (ov == bv && oi < bi))) {
+          bv = ov;
+          bi = oi;
+        }
+      }
+      if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
+    }
+    // Lane s < k checks cached slot s: a valid entry (in range, not repeated in the token) hits
+    // when its owner lane (e & 31) has marked it (bit e >> 5).
+    int e_slot = -1;
+    if (lane < k) {
+      const int e = cached[t * k + lane];
+      bool ok = e >= 0 && e < N;
+      for (int s2 = 0; ok && s2 < lane; ++s2)
+        if (cached[t * k + s2] == e) ok = false;
+      e_slot = ok ? e : -1;
+    }
+    const unsigned owner_mask = __shfl_sync(0xffffffffu, taken, e_slot >= 0 ? (e_slot & 31) : 0);
+    const bool hit = e_slot >= 0 && ((owner_mask >> (e_slot >> 5)) & 1u);
+    const int ov = __popc(__ballot_sync(0xffffffffu, hit));
+    if (lane == 0) {
+      atomicAdd(&sh_hist[k - ov], 1u);
+      atomicAdd(&sh_sum, static_cast<unsigned int>(ov));
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i <= k; i += blockDim.x)
+    if (sh_hist[i] != 0u) atomicAdd(&hist[i], static_cast<unsigned long long>(sh_hist[i]));
+  if (threadIdx.x == 0 && sh_sum != 0u)
+    atomicAdd(overlap_sum, static_cast<unsigned long long>(sh_sum));
+}
+
+// cache_h[c] = h[pos_c], cache_p[c] = logits[pos_c], pos_c = floor(c T / Tc); one warp per row.
+__global__ void __launch_bounds__(256)
+    feature_cache_kernel(const uint4* __restrict__ h, const float* __restrict__ logits,
+                         int64_t T, int64_t Tc, int row_vec, int N, int32_t* __restrict__ pos,
+                         uint4* __restrict__ cache_h, float* __restrict__ cache_p) {
+  pdl_wait();
+  pdl_trigger();
+  const int lane = threadIdx.x & 31;
+  const int64_t warp0 = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  for (int64_t c = warp0; c < Tc; c += nwarps) {
+    const int64_t p = (c * T) / Tc;
+    if (lane == 0) pos[c] = static_cast<int32_t>(p);
+    const uint4* src = h + p * row_vec;
+    uint4* dst = cache_h + c * row_vec;
+    for (int v = lane; v < row_vec; v += 32) dst[v] = __ldg(src + v);
+    if (logits != nullptr) {
+      const float* ls = logits + p * N;
+      float* ld = cache_p + c * N;
+      for (int v = lane; v < N; v += 32) ld[v] = __ldg(ls + v);
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_diagnostics(const float* rho, const int32_t* cached, int64_t T, int N, int k,
+                               int64_t* hist, int64_t* overlap_sum, cudaStream_t st) {
+  if (T == 0) return cudaSuccess;
+  const unsigned blocks = static_cast<unsigned>((T + kWarps - 1) / kWarps);
+  return launch_pdl(diagnostics_kernel, dim3(blocks), dim3(kWarps * 32), 0, st, 1, rho, cached,
+                    T, N, k, reinterpret_cast<unsigned long long*>(hist),
+                    reinterpret_cast<unsigned long long*>(overlap_sum));
+}
+
+cudaError_t launch_feature_cache(const void* h, const float* logits, int64_t T, int64_t Tc,
+                                 int d, int N, int esz, int32_t* pos, void* cache_h,
+                                 float* cache_p, int num_sms, cudaStream_t st) {
+  if (Tc == 0) return cudaSuccess;
+  int64_t blocks = (Tc + 7) / 8;
+  const int64_t cap = static_cast<int64_t>(num_sms) * 8;
+  if (blocks > cap) blocks = cap;
+  return launch_pdl(feature_cache_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, 1,
+                    static_cast<const uint4*>(h), logits, T, Tc, d * esz / 16, N, pos,
+                    static_cast<uint4*>(cache_h), cache_p);
+}
+
+}  // namespace pr2

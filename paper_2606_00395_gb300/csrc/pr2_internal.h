@@ -161,6 +161,13 @@ cudaError_t launch_loss_simt(const float* h_old, const float* p_old, const float
 cudaError_t launch_loss_grad_simt(const float* G, const float* h_old, int Tc, int d, int N,
                                   float* grad, cudaStream_t st);
 
+// ---- diagnostics and feature cache (diagnostics.cu) ---------------------------------------
+cudaError_t launch_diagnostics(const float* rho, const int32_t* cached, int64_t T, int N, int k,
+                               int64_t* hist, int64_t* overlap_sum, cudaStream_t st);
+cudaError_t launch_feature_cache(const void* h, const float* logits, int64_t T, int64_t Tc,
+                                 int d, int N, int esz, int32_t* pos, void* cache_h,
+                                 float* cache_p, int num_sms, cudaStream_t st);
+
 // ---- self test (api.cu) --------------------------------------------------------------------
 cudaError_t launch_wait_selftest(int32_t* status, int64_t timeout_ns, cudaStream_t st);
 

@@ -144,3 +144,25 @@ def test_predictor_loss_rejects_bad_arguments_on_the_host(lib):
     dms = B.dims(256, 2048, 128, 8, 768, flags=B.PR2_F_SYNC_STATUS | B.PR2_F_DELTA_LOSS)
     assert lib.pr2_predictor_loss(ctypes.byref(dms), *ok[1:], fake, ctypes.c_size_t(1 << 40),
                                   None, None) == 1
+
+
+def test_diagnostics_and_feature_cache_reject_bad_arguments(lib):
+    fake = ctypes.c_void_p(256)
+    dm = B.dims(64, 2048, 128, 8, 768)
+    assert lib.pr2_route_diagnostics(ctypes.byref(dm), fake, fake, None, fake, None) == 1
+    assert lib.pr2_route_diagnostics(ctypes.byref(dm), None, fake, fake, fake, None) == 1
+    assert lib.pr2_route_diagnostics(ctypes.byref(dm), ctypes.c_void_p(260), fake, fake, fake,
+                                     None) == 1
+    dm0 = B.dims(0, 2048, 128, 8, 768)
+    assert lib.pr2_route_diagnostics(ctypes.byref(dm0), None, None, fake, fake, None) == 0
+    # feature cache: T_c outside [0, T], missing buffers, half-given logits pair
+    assert lib.pr2_feature_cache_write(ctypes.byref(dm), 65, fake, fake, fake, fake, fake,
+                                       None) == 1
+    assert lib.pr2_feature_cache_write(ctypes.byref(dm), -1, fake, fake, fake, fake, fake,
+                                       None) == 1
+    assert lib.pr2_feature_cache_write(ctypes.byref(dm), 8, fake, fake, None, fake, fake,
+                                       None) == 1
+    assert lib.pr2_feature_cache_write(ctypes.byref(dm), 8, fake, fake, fake, fake, None,
+                                       None) == 1
+    assert lib.pr2_feature_cache_write(ctypes.byref(dm), 0, None, None, None, None, None,
+                                       None) == 0
