@@ -171,6 +171,84 @@ def host_layer(cfg, L):
 
 # ----------------------------------------------------------------------------------- pr2 arm
 
+def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
+    """The rows that widen the hot path, each timed alone on the device (CUDA events around the
+    call, L2 flushed before every call, median of ``iters``) against its own roofline:
+    the fixed-length feature-cache writer (Algorithm 2) for T_c = min(2048, T) rows (Table 4's
+    Qwen3 cache length), the predictive loss with its W_p gradient over that cache (Eq.
+    pr2_loss, Algorithm 3) and the route-tracking diagnostics of the rollout route against the
+    drifted current router (Sec. 5)."""
+    dev = "cuda"
+    Tc = min(2048, cfg.T)
+    idx, gates, logits = B.alloc_route(dm, logits=True)
+    B.check(B.pr2_route_predict(dm, L["x"], L["W_router"], L["W_pred"], idx, gates, logits),
+            "pr2_route_predict")
+    rho = torch.empty(cfg.T, cfg.N, dtype=torch.float32, device=dev)
+    rg = torch.empty_like(gates)
+    B.check(B.pr2_route_replay(dm, L["x"], W2, idx, rg, rho), "pr2_route_replay")
+    pos = torch.empty(Tc, dtype=torch.int32, device=dev)
+    ch = torch.empty(Tc, cfg.d, dtype=cfg.torch_dtype, device=dev)
+    cp = torch.empty(Tc, cfg.N, dtype=torch.float32, device=dev)
+    dml = B.dims(Tc, cfg.d, cfg.N, cfg.k, cfg.m, 0, cfg.dtype)
+    ws = B.alloc_loss_workspace(dml)
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    kl = torch.empty(Tc, dtype=torch.float32, device=dev)
+    grad = torch.empty(cfg.N, cfg.d, dtype=torch.float32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    hist = torch.zeros(cfg.k + 1, dtype=torch.int64, device=dev)
+    ov = torch.zeros(1, dtype=torch.int64, device=dev)
+
+    def timed(fn, pre=None):
+        evs = []
+        for i in range(iters + 3):
+            flush.fill_(i & 0xFF)
+            if pre is not None:
+                pre()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            evs.append((a, b))
+        torch.cuda.synchronize()
+        return statistics.median(a.elapsed_time(b) for a, b in evs[3:])
+
+    out = {}
+
+    def report(name, ms, w, **extra):
+        t_hbm = w.bytes / (pk["hbm"] * 1e9) * 1e3
+        t_tc = w.flops / (pk["bf16"] * 1e12) * 1e3
+        bound = "tensor" if t_tc > t_hbm else "hbm"
+        achieved = (w.flops / (ms * 1e-3) / 1e12) if bound == "tensor" else (
+            w.bytes / (ms * 1e-3) / 1e9)
+        out[name] = dict(ms=ms, bound=bound, achieved=achieved,
+                         peak=pk["bf16"] if bound == "tensor" else pk["hbm"],
+                         unit="TFLOP/s" if bound == "tensor" else "GB/s",
+                         frac=max(t_hbm, t_tc) / ms, algorithmic_bytes=w.bytes,
+                         algorithmic_flops=w.flops, **extra)
+
+    ms = timed(lambda: B.check(B.pr2_feature_cache_write(dm, Tc, L["x"], logits, pos, ch, cp),
+                               "pr2_feature_cache_write"))
+    report("feature_cache_write", ms, cost.feature_cache_work(Tc, cfg.d, cfg.N, cfg.dtype), Tc=Tc)
+    ms = timed(lambda: B.check(B.pr2_predictor_loss(dml, ch, cp, L["W_pred"], rho, loss, grad,
+                                                    pos=pos, kl_tok=kl, workspace=ws,
+                                                    status=status), "pr2_predictor_loss"))
+    report("predictor_loss", ms, cost.predictor_loss_work(Tc, cfg.d, cfg.N, cfg.dtype), Tc=Tc,
+           loss=float(loss.item()))
+
+    def zero():
+        hist.zero_()
+        ov.zero_()
+    ms = timed(lambda: B.check(B.pr2_route_diagnostics(dm, rho, idx, hist, ov),
+                               "pr2_route_diagnostics"), pre=zero)
+    report("route_diagnostics", ms, cost.route_diagnostics_work(cfg.T, cfg.N, cfg.k),
+           topk_agreement=int(ov.item()) / (cfg.T * cfg.k),
+           deviation_hist=[int(x) for x in hist.tolist()])
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())} in the extra rows")
+    return out
+
+
 def run_pr2(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     dist = None
@@ -330,6 +408,8 @@ def run_pr2(args, rank, world, local_rank):
                     algorithmic=("flops" if dk["bound"] == "tensor" else "bytes"),
                     per_launch_units=f"{F} token-expert rows x (d={cfg.d}, m={cfg.m})")
 
+    extras = measure_extras(cfg, L, W2, dm, flush, pk)
+
     # ---- end to end through the public API with host buffers
     xh = torch.empty(cfg.T, cfg.d, dtype=cfg.torch_dtype, pin_memory=True)
     xh.copy_(L["x"].cpu())
@@ -370,7 +450,7 @@ def run_pr2(args, rank, world, local_rank):
                            replay_tokens_per_s=cfg.T / (mean["layer_replay"] / 1e3),
                            note="from the per-kernel breakdown pass (stage events)"),
                 breakdown_ms_per_step=mean["step"],
-                kernels=kernels, near_tie_tokens_per_step=near_per_step)
+                kernels=kernels, near_tie_tokens_per_step=near_per_step, extras=extras)
 
     if rank == 0 and not args.no_cpu_baseline:
         Lh = host_layer(cfg, L)

@@ -86,3 +86,23 @@ def combine_work(T: int, d: int, k: int, n_shared: int = 0, dtype: str = "bf16")
     """out[t] = sum_s g[t,s] Y[inv[t,s]] (+ shared rows): read Y, gates, inv; write out."""
     e = _esz(dtype)
     return KernelWork(T * k * d * e + T * k * 8 + T * n_shared * d * e + T * d * e, 0)
+
+
+def predictor_loss_work(Tc: int, d: int, N: int, dtype: str = "bf16") -> KernelWork:
+    """Eq. pr2_loss with its W_p gradient over T_c cached rows: read h_old, p_old, the teacher
+    rows and W_p once, write the gradient and the per-token KL; FLOPs of the two products
+    b = h_old W_p^T and (dKL/dz)^T h_old."""
+    e = _esz(dtype)
+    b = Tc * d * e + 2 * Tc * N * 4 + N * d * e + N * d * 4 + Tc * 4
+    return KernelWork(b, 2 * Tc * d * N + 2 * N * d * Tc)
+
+
+def route_diagnostics_work(T: int, N: int, k: int) -> KernelWork:
+    """Top-k agreement / deviation histogram: read rho [T, N] fp32 and the cached route."""
+    return KernelWork(T * N * 4 + T * k * 4, 0)
+
+
+def feature_cache_work(Tc: int, d: int, N: int, dtype: str = "bf16") -> KernelWork:
+    """Feature-cache writer: read and write T_c rows of h and p_old, write the positions."""
+    e = _esz(dtype)
+    return KernelWork(2 * Tc * (d * e + N * 4) + Tc * 4, 0)

@@ -32,3 +32,17 @@ def test_kernel_work_counts_each_tensor_once():
     g = cost.expert_gate_up_work(32768, 2048, 768, 128)
     dn = cost.expert_down_work(32768, 2048, 768, 128)
     assert g.flops + dn.flops == 6 * 4096 * 8 * 2048 * 768
+
+
+def test_tracking_and_loss_work_match_table4_sizes():
+    """The feature-cache writer moves each cached byte of Table 4 twice (read and write), one
+    layer at a time; the predictive loss does the predictor projection and its transpose."""
+    row = next(r for r in GOLDEN["rows"] if r["model"].startswith("Qwen3"))
+    Tc, d, N = row["T_c"], row["d"], row["N"]
+    fc = cost.feature_cache_work(Tc, d, N)
+    assert fc.bytes == 2 * cost.feature_cache_bytes(Tc, 1, d, N) + 4 * Tc
+    lw = cost.predictor_loss_work(Tc, d, N)
+    assert lw.flops == 2 * Tc * cost.predictor_flops_per_token(1, d, N)
+    assert lw.bytes > Tc * 2 * d
+    dg = cost.route_diagnostics_work(4096, N, row["k"])
+    assert dg.bytes == 4096 * (4 * N + 4 * row["k"])
