@@ -226,6 +226,32 @@ pr2_status pr2_feature_cache_write(const pr2_dims* dims, int64_t T_c, const void
                                    const float* logits_old, int32_t* pos, void* cache_h,
                                    float* cache_p, void* stream);
 
+/*
+ * Multi-layer rollout decode: L Pr^2 MoE layers in rollout mode applied in sequence to one
+ * batch of T tokens, as the route-recording phase runs them layer after layer (Algorithm 2 for
+ * l = 1..L: predict the route, record it and the features, compute o_old^(l); App. "Pr^3"
+ * uses the same rollout-engine pass).  Between layers the residual stream
+ * h^(l+1) = h^(l) + o_old^(l) (rounded once to dims->dtype) stands in for the rest of the
+ * transformer block; attention and normalisation are outside this library.
+ *  h [T, d] dims->dtype: h^(1) on entry, h^(L+1) on return (updated in place).
+ *  Weights stacked by layer: W_router, W_pred [L, N, d]; W_gate, W_up [L, N, m, d];
+ *    W_down [L, N, d, m]; shared experts Ws_gate, Ws_up [L, n_shared, m, d],
+ *    Ws_down [L, n_shared, d, m] (NULL iff n_shared == 0).
+ *  Outputs per layer, as pr2_route_predict writes them: idx [L, T, k], gates [L, T, k],
+ *    logits_old [L, T, N] (nullable: the feature-cache logits p_old); near_tie (nullable) counts
+ *    over all layers.
+ *  workspace: pr2_moe_workspace_bytes(dims) bytes, reused by every layer.
+ * Every step is an asynchronous launch on `stream` (no host synchronisation unless
+ * PR2_F_SYNC_STATUS), so the whole loop can be captured into a CUDA graph by the caller and
+ * replayed; results equal those of L pairs of pr2_route_predict / pr2_moe_forward calls.
+ */
+pr2_status pr2_rollout_layers(const pr2_dims* dims, int32_t L, void* h, const void* W_router,
+                              const void* W_pred, const void* W_gate, const void* W_up,
+                              const void* W_down, const void* Ws_gate, const void* Ws_up,
+                              const void* Ws_down, int32_t* idx, float* gates,
+                              float* logits_old, int64_t* near_tie, void* workspace,
+                              size_t ws_bytes, int32_t* status_dev, void* stream);
+
 /* Static, human-readable name of a status code. */
 const char* pr2_strerror(pr2_status s);
 

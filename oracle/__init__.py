@@ -15,6 +15,8 @@ Functions (each cites the passage it follows in the C source):
   delta-matching variant of the appendix ablation
 * ``route_diagnostics`` - top-k agreement and the deviation histogram (Sec. 5)
 * ``feature_cache``  - the fixed-length feature cache of Algorithm 2 (evenly spaced positions)
+* ``rollout_layers`` - Algorithm 2 over L stacked layers with the residual stream (composition
+  of ``route_predict`` and ``moe_forward``)
 
 Parity status: every function is pinned by the CPU tests in ``tests/test_oracle_pins.py``.
 """
@@ -273,3 +275,54 @@ def feature_cache(h, logits, Tc: int, lib=None):
     if isinstance(h, torch.Tensor):
         hc = hc.view(h.dtype)
     return dict(pos=pos[:Tc], h=hc, p=cp[:Tc])
+
+
+def _round_to(x: np.ndarray, dtype) -> torch.Tensor:
+    """fp64 values rounded once (to nearest, ties to even) to ``dtype``, as a tensor.  bf16 is
+    rounded straight from the fp64 bit pattern (no intermediate fp32 rounding): keep the top 7
+    of the 52 mantissa bits, round on the other 45, carry into the exponent."""
+    x = np.ascontiguousarray(x, dtype=np.float64)
+    if dtype != torch.bfloat16:
+        return torch.from_numpy(x).to(dtype)
+    b = x.view(np.uint64)
+    sign = (b >> np.uint64(63)) & np.uint64(1)
+    exp = ((b >> np.uint64(52)) & np.uint64(0x7FF)).astype(np.int64)
+    man = b & np.uint64((1 << 52) - 1)
+    keep = (man >> np.uint64(45)).astype(np.int64)
+    rem = (man & np.uint64((1 << 45) - 1)).astype(np.int64)
+    half = 1 << 44
+    keep = keep + ((rem > half) | ((rem == half) & ((keep & 1) == 1))).astype(np.int64)
+    e32 = exp - 1023 + 127 + (keep >> 7)
+    keep &= 0x7F
+    zero = exp == 0
+    if np.any(~zero & ((e32 < 1) | (e32 > 254))):
+        raise ValueError("value outside the normal bf16 range")
+    bits = (sign.astype(np.int64) << 15) | np.where(zero, 0, (e32 << 7) | keep)
+    return torch.from_numpy(bits.astype(np.uint16).view(np.int16)).view(torch.bfloat16)
+
+
+def rollout_layers(h, layers, k: int, lib=None):
+    """Algorithm 2 applied to layers l = 1..L in sequence (the route-recording pass of a stack of
+    MoE layers): at each layer the rollout route and output of Eqs. pr2_predict / pr2_route /
+    pr2_old_output, then the residual stream h <- round(h + o_old) in h's dtype (the layer's
+    output is stored once in the layer dtype).  ``layers`` is a list of dicts with W_router,
+    W_pred, W_gate, W_up, W_down (and optionally Ws_*).  Returns dict(h [T,d] tensor in h's
+    dtype, idx [L,T,k], gates [L,T,k], logits [L,T,N], margin [L,T] (rho_(k) - rho_(k+1)),
+    min_gap [L,T] (smallest gap between consecutive ones of the top k+1 probabilities, which
+    also bounds how near the slot order is to a tie))."""
+    cur = h.detach().to("cpu").contiguous()
+    idx, gates, logits, margin, min_gap = [], [], [], [], []
+    for lw in layers:
+        r = route_predict(cur, lw["W_router"], lw["W_pred"], k, lib=lib)
+        o = moe_forward(cur, r["idx"], r["gates"], lw["W_gate"], lw["W_up"], lw["W_down"],
+                        lw.get("Ws_gate"), lw.get("Ws_up"), lw.get("Ws_down"), lib=lib)
+        cur = _round_to(cur.double().numpy() + o, cur.dtype)
+        idx.append(r["idx"])
+        gates.append(r["gates"])
+        logits.append(r["logits"])
+        margin.append(r["margin"])
+        tv = r["top_vals"][:, : min(k + 1, r["logits"].shape[1])]
+        min_gap.append(np.min(tv[:, :-1] - tv[:, 1:], axis=1) if tv.shape[1] > 1
+                       else np.full(tv.shape[0], np.inf))
+    return dict(h=cur, idx=np.stack(idx), gates=np.stack(gates), logits=np.stack(logits),
+                margin=np.stack(margin), min_gap=np.stack(min_gap))

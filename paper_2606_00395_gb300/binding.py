@@ -104,6 +104,9 @@ def load() -> ctypes.CDLL:
         lib.pr2_route_diagnostics.restype = ctypes.c_int
         lib.pr2_feature_cache_write.argtypes = [D, I64, P, P, P, P, P, P]
         lib.pr2_feature_cache_write.restype = ctypes.c_int
+        lib.pr2_rollout_layers.argtypes = [D, I32, P, P, P, P, P, P, P, P, P, P, P, P, P, P,
+                                           ctypes.c_size_t, P, P]
+        lib.pr2_rollout_layers.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -196,6 +199,20 @@ def pr2_feature_cache_write(dm: Dims, Tc: int, h, logits_old, pos, cache_h, cach
                             stream=None) -> int:
     return load().pr2_feature_cache_write(ctypes.byref(dm), int(Tc), _p(h), _p(logits_old),
                                           _p(pos), _p(cache_h), _p(cache_p), _s(stream))
+
+
+def pr2_rollout_layers(dm: Dims, L: int, h, W_router, W_pred, W_gate, W_up, W_down, idx, gates,
+                       Ws_gate=None, Ws_up=None, Ws_down=None, logits_old=None, near_tie=None,
+                       workspace=None, ws_bytes=None, status=None, stream=None) -> int:
+    """L rollout layers in sequence with the residual stream updated in ``h`` (in place);
+    weights stacked by layer, per-layer routes in ``idx``/``gates`` [L, T, k]."""
+    if ws_bytes is None:
+        ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    return load().pr2_rollout_layers(ctypes.byref(dm), int(L), _p(h), _p(W_router), _p(W_pred),
+                                     _p(W_gate), _p(W_up), _p(W_down), _p(Ws_gate), _p(Ws_up),
+                                     _p(Ws_down), _p(idx), _p(gates), _p(logits_old),
+                                     _p(near_tie), _p(workspace), ctypes.c_size_t(ws_bytes),
+                                     _p(status), _s(stream))
 
 
 # ---- allocation helpers (plain torch.empty on the caller's device) ---------------------------

@@ -362,12 +362,20 @@ size_t pr2_moe_workspace_bytes(const pr2_dims* dims) {
   return carve(*dims, nullptr).total;
 }
 
-pr2_status pr2_moe_forward(const pr2_dims* dims, const void* h, const int32_t* idx,
-                           const float* gates, const void* W_gate, const void* W_up,
-                           const void* W_down, const void* Ws_gate, const void* Ws_up,
-                           const void* Ws_down, void* out, int32_t* counts, int32_t* perm,
-                           void* workspace, size_t ws_bytes, int32_t* status_dev,
-                           const pr2_stage_events* events, void* stream) {
+}  // extern "C"
+
+namespace pr2 {
+namespace {
+
+// The layer forward of pr2_moe_forward; `residual` (nullable, [T, d] in the layer dtype, may
+// alias `out`) is added to the combined output.
+pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* idx,
+                            const float* gates, const void* W_gate, const void* W_up,
+                            const void* W_down, const void* Ws_gate, const void* Ws_up,
+                            const void* Ws_down, void* out, const void* residual,
+                            int32_t* counts, int32_t* perm, void* workspace, size_t ws_bytes,
+                            int32_t* status_dev, const pr2_stage_events* events,
+                            void* stream) {
   pr2_status s = check_dims(dims);
   if (s != PR2_OK) return s;
   const pr2_dims& dm = *dims;
@@ -458,7 +466,7 @@ pr2_status pr2_moe_forward(const pr2_dims* dims, const void* h, const int32_t* i
   if (err != cudaSuccess) return PR2_ERR_CUDA;
 
   CombineArgs ca{w.ybuf, dm.n_shared > 0 ? w.ys : nullptr, w.inv, gates, dm.T, dm.k, dm.d,
-                 dm.n_shared, dm.dtype == PR2_BF16 ? 1 : 0, out};
+                 dm.n_shared, dm.dtype == PR2_BF16 ? 1 : 0, out, residual};
   err = launch_combine(ca, num_sms, st);
   mark(events ? events->end : nullptr);
   if (err == cudaSuccess && counts != nullptr)
@@ -466,6 +474,64 @@ pr2_status pr2_moe_forward(const pr2_dims* dims, const void* h, const int32_t* i
   if (err == cudaSuccess && perm != nullptr)
     err = cudaMemcpyAsync(perm, w.perm, sizeof(int32_t) * F, cudaMemcpyDeviceToDevice, st);
   return finish(err, dm.flags, status, st);
+}
+
+}  // namespace
+}  // namespace pr2
+
+extern "C" {
+
+pr2_status pr2_moe_forward(const pr2_dims* dims, const void* h, const int32_t* idx,
+                           const float* gates, const void* W_gate, const void* W_up,
+                           const void* W_down, const void* Ws_gate, const void* Ws_up,
+                           const void* Ws_down, void* out, int32_t* counts, int32_t* perm,
+                           void* workspace, size_t ws_bytes, int32_t* status_dev,
+                           const pr2_stage_events* events, void* stream) {
+  return moe_forward_impl(dims, h, idx, gates, W_gate, W_up, W_down, Ws_gate, Ws_up, Ws_down,
+                          out, nullptr, counts, perm, workspace, ws_bytes, status_dev, events,
+                          stream);
+}
+
+pr2_status pr2_rollout_layers(const pr2_dims* dims, int32_t L, void* h, const void* W_router,
+                              const void* W_pred, const void* W_gate, const void* W_up,
+                              const void* W_down, const void* Ws_gate, const void* Ws_up,
+                              const void* Ws_down, int32_t* idx, float* gates,
+                              float* logits_old, int64_t* near_tie, void* workspace,
+                              size_t ws_bytes, int32_t* status_dev, void* stream) {
+  pr2_status s = check_dims(dims);
+  if (s != PR2_OK) return s;
+  const pr2_dims& dm = *dims;
+  if (L < 1) return PR2_ERR_INVALID_ARG;
+  if ((dm.flags & PR2_F_SYNC_STATUS) && status_dev == nullptr) return PR2_ERR_INVALID_ARG;
+  if (dm.T == 0) return PR2_OK;
+  if (h == nullptr || W_router == nullptr || W_pred == nullptr || W_gate == nullptr ||
+      W_up == nullptr || W_down == nullptr || idx == nullptr || gates == nullptr)
+    return PR2_ERR_INVALID_ARG;
+  const size_t es = esize(dm);
+  const size_t r_sz = (size_t)dm.N * dm.d * es;            // one layer's router / predictor
+  const size_t gu_sz = (size_t)dm.N * dm.m * dm.d * es;    // gate or up (and down) stack
+  const size_t sgu_sz = (size_t)dm.n_shared * dm.m * dm.d * es;
+  auto base = [](const void* p, size_t off) -> const void* {
+    return p == nullptr ? nullptr : static_cast<const uint8_t*>(p) + off;
+  };
+  // Each layer's status goes to the caller's word (or the forward's own), read once at the end.
+  const uint32_t lf = dm.flags & ~PR2_F_SYNC_STATUS;
+  pr2_dims dl = dm;
+  dl.flags = lf;
+  for (int32_t l = 0; l < L; ++l) {
+    int32_t* idx_l = idx + (size_t)l * dm.T * dm.k;
+    float* gates_l = gates + (size_t)l * dm.T * dm.k;
+    float* logits_l = logits_old ? logits_old + (size_t)l * dm.T * dm.N : nullptr;
+    s = pr2_route_predict(&dl, h, base(W_router, l * r_sz), base(W_pred, l * r_sz), idx_l,
+                          gates_l, logits_l, near_tie, status_dev, stream);
+    if (s != PR2_OK) return s;
+    s = moe_forward_impl(&dl, h, idx_l, gates_l, base(W_gate, l * gu_sz), base(W_up, l * gu_sz),
+                         base(W_down, l * gu_sz), base(Ws_gate, l * sgu_sz),
+                         base(Ws_up, l * sgu_sz), base(Ws_down, l * sgu_sz), h, h, nullptr,
+                         nullptr, workspace, ws_bytes, status_dev, nullptr, stream);
+    if (s != PR2_OK) return s;
+  }
+  return finish(cudaSuccess, dm.flags, status_dev, static_cast<cudaStream_t>(stream));
 }
 
 const char* pr2_strerror(pr2_status s) {

@@ -12,7 +12,8 @@
 //               perm[offsets[e] + r] = f, inv[f] = its position (-1 for an invalid slot).
 //   4. gather - X[p, :] = h[perm[p] / k, :], 16-byte vectors, one warp per row.
 // Combine (the sums of Eqs. pr2_old_output / pr2_output):
-//   out[t, :] = sum_s gates[t,s] * Y[inv[t*k+s], :] + sum_j Ys[j, t, :], fp32 accumulation.
+//   out[t, :] = sum_s gates[t,s] * Y[inv[t*k+s], :] + sum_j Ys[j, t, :], fp32 accumulation,
+//   plus, when given, a residual row r[t, :] (the multi-layer loop's h_l; may alias out).
 #include "pr2_device.cuh"
 #include "pr2_internal.h"
 
@@ -231,7 +232,7 @@ template <typename T, int V, int KMAX>  // V elements per 16-byte vector, k <= K
 __global__ void __launch_bounds__(256)
     combine_kernel(const T* __restrict__ Y, const T* __restrict__ Ys,
                    const int32_t* __restrict__ inv, const float* __restrict__ gates, int64_t Tn,
-                   int k, int d, int n_shared, T* __restrict__ out) {
+                   int k, int d, int n_shared, const T* residual, T* out) {
   pdl_wait();
   pdl_trigger();
   const int lane = threadIdx.x & 31;
@@ -262,6 +263,12 @@ __global__ void __launch_bounds__(256)
       float acc[V];
 #pragma unroll
       for (int j = 0; j < V; ++j) acc[j] = 0.f;
+      if (residual != nullptr) {  // read before the same thread overwrites it (in place)
+        const uint4 r = reinterpret_cast<const uint4*>(residual + t * d)[c];
+        const T* v = reinterpret_cast<const T*>(&r);
+#pragma unroll
+        for (int j = 0; j < V; ++j) acc[j] = to_f32<T>(v[j]);
+      }
 #pragma unroll
       for (int s = 0; s < KMAX; ++s) {
         if (pos[s] < 0) continue;
@@ -327,18 +334,20 @@ cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st) {
     auto* Y = static_cast<const __nv_bfloat16*>(a.Y);
     auto* Ys = static_cast<const __nv_bfloat16*>(a.Ys);
     auto* out = static_cast<__nv_bfloat16*>(a.out);
+    auto* res = static_cast<const __nv_bfloat16*>(a.residual);
     return a.k <= 8 ? launch_pdl(combine_kernel<__nv_bfloat16, 8, 8>, grid, block, 0, st, 1, Y,
-                                 Ys, a.inv, a.gates, a.T, a.k, a.d, a.n_shared, out)
+                                 Ys, a.inv, a.gates, a.T, a.k, a.d, a.n_shared, res, out)
                     : launch_pdl(combine_kernel<__nv_bfloat16, 8, 32>, grid, block, 0, st, 1, Y,
-                                 Ys, a.inv, a.gates, a.T, a.k, a.d, a.n_shared, out);
+                                 Ys, a.inv, a.gates, a.T, a.k, a.d, a.n_shared, res, out);
   }
   auto* Y = static_cast<const float*>(a.Y);
   auto* Ys = static_cast<const float*>(a.Ys);
   auto* out = static_cast<float*>(a.out);
+  auto* res = static_cast<const float*>(a.residual);
   return a.k <= 8 ? launch_pdl(combine_kernel<float, 4, 8>, grid, block, 0, st, 1, Y, Ys, a.inv,
-                               a.gates, a.T, a.k, a.d, a.n_shared, out)
+                               a.gates, a.T, a.k, a.d, a.n_shared, res, out)
                   : launch_pdl(combine_kernel<float, 4, 32>, grid, block, 0, st, 1, Y, Ys, a.inv,
-                               a.gates, a.T, a.k, a.d, a.n_shared, out);
+                               a.gates, a.T, a.k, a.d, a.n_shared, res, out);
 }
 
 }  // namespace pr2

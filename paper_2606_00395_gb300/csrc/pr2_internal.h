@@ -115,6 +115,7 @@ struct CombineArgs {
   int64_t T;
   int k, d, n_shared, bf16;
   void* out;            // [T, d]
+  const void* residual; // [T, d] added to the sum (nullable); may equal `out`
 };
 cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st);
 

@@ -166,3 +166,25 @@ def test_diagnostics_and_feature_cache_reject_bad_arguments(lib):
                                        None) == 1
     assert lib.pr2_feature_cache_write(ctypes.byref(dm), 0, None, None, None, None, None,
                                        None) == 0
+
+
+def test_rollout_layers_rejects_bad_arguments(lib):
+    fake = ctypes.c_void_p(256)
+    dm = B.dims(64, 2048, 128, 8, 768)
+    ws = B.pr2_moe_workspace_bytes(dm)
+    # dims, L, h, W_router, W_pred, W_gate, W_up, W_down, Ws_* (3), idx, gates, logits, near_tie
+    base = [ctypes.byref(dm), ctypes.c_int32(2), fake, fake, fake, fake, fake, fake, None, None,
+            None, fake, fake, None, None]
+    bad_L = list(base)
+    bad_L[1] = ctypes.c_int32(0)
+    assert lib.pr2_rollout_layers(*bad_L, fake, ctypes.c_size_t(ws), None, None) == 1
+    no_idx = list(base)
+    no_idx[11] = None
+    assert lib.pr2_rollout_layers(*no_idx, fake, ctypes.c_size_t(ws), None, None) == 1
+    no_h = list(base)
+    no_h[2] = None
+    assert lib.pr2_rollout_layers(*no_h, fake, ctypes.c_size_t(ws), None, None) == 1
+    dms = B.dims(64, 2048, 128, 8, 768, flags=B.PR2_F_SYNC_STATUS)
+    sync = list(base)
+    sync[0] = ctypes.byref(dms)
+    assert lib.pr2_rollout_layers(*sync, fake, ctypes.c_size_t(ws), None, None) == 1

@@ -451,3 +451,38 @@ def test_feature_cache_evenly_spaced_rows(Tc):
     assert np.all(np.diff(pos) >= 1) and pos[-1] <= T - 1
     assert torch.equal(r["h"], h[torch.from_numpy(pos).long()])
     assert np.array_equal(r["p"], lg.numpy()[pos])
+
+
+# ---- Algorithm 2 over stacked layers (residual stream) ---------------------------------------
+
+def test_bf16_rounding_of_the_residual_stream_is_round_to_nearest_even():
+    x = np.array([1 + 2.0 ** -8, 1 + 3 * 2.0 ** -8, 1 + 2.0 ** -8 + 2.0 ** -40, -0.0, 0.0,
+                  -(1 + 2.0 ** -8 + 2.0 ** -40), 3.0 * 2.0 ** -20])
+    got = oracle._round_to(x, torch.bfloat16).float().numpy()
+    want = np.array([1.0, 1 + 2.0 ** -6, 1 + 2.0 ** -7, 0.0, 0.0, -(1 + 2.0 ** -7),
+                     3.0 * 2.0 ** -20])
+    assert np.array_equal(got, want)
+    r = np.random.default_rng(1).standard_normal(4096).astype(np.float32).astype(np.float64)
+    assert torch.equal(oracle._round_to(r, torch.bfloat16), torch.from_numpy(r).float().bfloat16())
+
+
+def test_rollout_layers_compose_single_layers():
+    cfg = synth.LayerConfig("t", T=16, d=16, N=4, k=2, m=8, dtype="fp32")
+    layers = [synth.make_layer(cfg, seed=20 + l) for l in range(3)]
+    h0 = layers[0]["x"]
+    r = oracle.rollout_layers(h0, layers, 2)
+    cur = h0.double().numpy()
+    for l, lw in enumerate(layers):
+        one = oracle.route_predict(torch.from_numpy(cur).float(), lw["W_router"], lw["W_pred"], 2)
+        assert np.array_equal(one["idx"], r["idx"][l])
+        o = oracle.moe_forward(torch.from_numpy(cur).float(), one["idx"], one["gates"],
+                               lw["W_gate"], lw["W_up"], lw["W_down"])
+        cur = (cur + o).astype(np.float32).astype(np.float64)
+    assert np.array_equal(r["h"].numpy(), cur.astype(np.float32))
+    # zero up-projections: every layer adds 0, the stream is unchanged, routes stay those of h0
+    zl = [dict(lw, W_up=torch.zeros_like(lw["W_up"])) for lw in layers]
+    z = oracle.rollout_layers(h0, zl, 2)
+    assert torch.equal(z["h"], h0)
+    for l, lw in enumerate(zl):
+        assert np.array_equal(z["idx"][l],
+                              oracle.route_predict(h0, lw["W_router"], lw["W_pred"], 2)["idx"])
