@@ -244,6 +244,65 @@ def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
     report("route_diagnostics", ms, cost.route_diagnostics_work(cfg.T, cfg.N, cfg.k),
            topk_agreement=int(ov.item()) / (cfg.T * cfg.k),
            deviation_hist=[int(x) for x in hist.tolist()])
+
+    # Multi-layer rollout decode (Algorithm 2 over L layers): a 256-token decode batch through
+    # L = 4 layers of this shape (the layer's weights repeated per layer, each layer streaming
+    # its own 1.2 GB copy), one pr2_rollout_layers call, eager and replayed from a CUDA graph.
+    Ld, Td = 4, min(256, cfg.T)
+    ddm = B.dims(Td, cfg.d, cfg.N, cfg.k, cfg.m, cfg.n_shared, cfg.dtype)
+    keys = ["W_router", "W_pred", "W_gate", "W_up", "W_down"]
+    keys += ["Ws_gate", "Ws_up", "Ws_down"] if cfg.n_shared else []
+    Ws = {k: torch.stack([L[k]] * Ld).contiguous() for k in keys}
+    h0 = L["x"][:Td].clone()
+    hd = h0.clone()
+    didx = torch.empty(Ld, Td, cfg.k, dtype=torch.int32, device=dev)
+    dgates = torch.empty(Ld, Td, cfg.k, dtype=torch.float32, device=dev)
+    dlog = torch.empty(Ld, Td, cfg.N, dtype=torch.float32, device=dev)
+    dws = B.alloc_workspace(ddm)
+
+    def loop(stream=None):
+        return B.pr2_rollout_layers(ddm, Ld, hd, Ws["W_router"], Ws["W_pred"], Ws["W_gate"],
+                                    Ws["W_up"], Ws["W_down"], didx, dgates,
+                                    Ws_gate=Ws.get("Ws_gate"), Ws_up=Ws.get("Ws_up"),
+                                    Ws_down=Ws.get("Ws_down"), logits_old=dlog,
+                                    workspace=dws, status=status, stream=stream)
+
+    eager_ms = timed(lambda: B.check(loop(), "pr2_rollout_layers"), pre=lambda: hd.copy_(h0))
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=side):
+        B.check(loop(side), "pr2_rollout_layers (capture)")
+    graph_ms = timed(graph.replay, pre=lambda: hd.copy_(h0))
+    per_layer = [cost.route_predict_work(Td, cfg.d, cfg.N, cfg.k, cfg.dtype, True),
+                 cost.dispatch_work(Td, cfg.d, cfg.k, cfg.dtype),
+                 cost.expert_gate_up_work(Td * cfg.k, cfg.d, cfg.m, cfg.N, cfg.dtype),
+                 cost.expert_down_work(Td * cfg.k, cfg.d, cfg.m, cfg.N, cfg.dtype),
+                 cost.combine_work(Td, cfg.d, cfg.k, cfg.n_shared, cfg.dtype)]
+    work = cost.KernelWork(Ld * sum(w.bytes for w in per_layer),
+                           Ld * sum(w.flops for w in per_layer))
+    report("decode_loop_graph", graph_ms, work, layers=Ld, T=Td, eager_ms=eager_ms,
+           tokens_per_s=Td / (graph_ms * 1e-3))
+    del Ws, graph
+
+    # Pr^3 step (App. "Predictive Rollout Routing Replay"): rollout with the predicted route,
+    # the log-prob pass replaying it with the snapshot router, the gradient pass replaying it
+    # with the current (drifted) router; T tokens, step-boundary events only.
+    o1 = torch.empty(cfg.T, cfg.d, dtype=cfg.torch_dtype, device=dev)
+    wsl = B.alloc_workspace(dm)
+
+    def pr3():
+        B.check(B.pr2_route_predict(dm, L["x"], L["W_router"], L["W_pred"], idx, gates, logits),
+                "pr2_route_predict")
+        sh = (L["Ws_gate"], L["Ws_up"], L["Ws_down"])
+        B.check(B.pr2_moe_forward(dm, L["x"], idx, gates, L["W_gate"], L["W_up"], L["W_down"],
+                                  *sh, o1, workspace=wsl), "pr2_moe_forward")
+        for Wr in (L["W_router"], W2):
+            B.check(B.pr2_route_replay(dm, L["x"], Wr, idx, rg, None), "pr2_route_replay")
+            B.check(B.pr2_moe_forward(dm, L["x"], idx, rg, L["W_gate"], L["W_up"], L["W_down"],
+                                      *sh, o1, workspace=wsl), "pr2_moe_forward")
+    ms = timed(pr3)
+    out["pr3_step"] = dict(ms=ms, tokens_per_s=cfg.T / (ms * 1e-3), passes=3, T=cfg.T)
     if int(status.item()) != 0:
         raise RuntimeError(f"device status {int(status.item())} in the extra rows")
     return out
