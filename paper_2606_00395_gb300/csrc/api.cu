@@ -331,8 +331,11 @@ pr2_status pr2_route_diagnostics(const pr2_dims* dims, const float* rho, const i
   if (hist == nullptr || overlap_sum == nullptr) return PR2_ERR_INVALID_ARG;
   if (dm.T == 0) return PR2_OK;
   if (rho == nullptr || idx_cached == nullptr || !aligned16(rho)) return PR2_ERR_INVALID_ARG;
+  const int num_sms = num_sms_of_current_device();
+  if (num_sms <= 0) return PR2_ERR_CUDA;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  return finish(launch_diagnostics(rho, idx_cached, dm.T, dm.N, dm.k, hist, overlap_sum, st),
+  return finish(launch_diagnostics(rho, idx_cached, dm.T, dm.N, dm.k, hist, overlap_sum, num_sms,
+                                   st),
                 dm.flags & ~PR2_F_SYNC_STATUS, nullptr, st);
 }
 

@@ -1,11 +1,14 @@
 // Route-tracking diagnostics (Sec. 5 "Top-k Agreement and Route KL", "Deviation Tails") and the
 // fixed-length feature-cache writer (Algorithm 2, App. "uniform sub-sampling").
 //
-// Diagnostics: one warp per token.  Lane l holds rho[t, 32 j + l]; k rounds of warp argmax
-// (largest value, lower expert on equal values, as TopK of Eq. pr2_route) mark I_t = TopK(rho_t,
-// k); overlap_t = |Î_t ∩ I_t| counts the cached entries (in range, not repeated) that are
-// marked.  hist[k - overlap_t] and sum_t overlap_t are accumulated with 64-bit integer atomics
-// (order-independent, so exact and deterministic).
+// Diagnostics: one warp per token.  Lane l holds rho[t, 32 j + l].  A cached expert e lies in
+// I_t = TopK(rho_t, k) (largest values, the lower expert first on equal values, as TopK of Eq.
+// pr2_route) exactly when fewer than k experts beat it, where j beats e if rho_j > rho_e or
+// rho_j = rho_e and j < e; the warp counts the experts that beat each cached entry with ballots.
+// overlap_t = |Î_t ∩ I_t| counts the cached entries (in range, not repeated) that pass.  hist[k - overlap_t] and sum_t overlap_t are accumulated per block in shared memory
+// and then with 64-bit integer atomics (order-independent, so exact and deterministic); the
+// grid is at most two blocks per SM, each looping over tokens, so that the k + 2 global
+// counters see few atomics.
 // Feature cache: row c of the cache is row pos_c = floor(c T / T_c) of the batch; one warp per
 // cached row copies h (16-byte vectors) and the fp32 router logits.
 #include "pr2_device.cuh"
@@ -15,7 +18,7 @@ namespace pr2 {
 namespace {
 
 constexpr int kPerLane = kMaxExperts / 32;
-constexpr int kWarps = 8;
+constexpr int kWarps = 16;
 
 __global__ void __launch_bounds__(kWarps * 32)
     diagnostics_kernel(const float* __restrict__ rho, const int32_t* __restrict__ cached,
@@ -29,8 +32,9 @@ __global__ void __launch_bounds__(kWarps * 32)
   if (threadIdx.x == 0) sh_sum = 0u;
   __syncthreads();
   const int lane = threadIdx.x & 31;
-  const int64_t t = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
-  if (t < T) {
+  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * kWarps;
+  for (int64_t t = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5); t < T;
+       t += nwarps) {
     const float* row = rho + t * N;
     float v[kPerLane];
 #pragma unroll
@@ -38,42 +42,25 @@ __global__ void __launch_bounds__(kWarps * 32)
       const int e = j * 32 + lane;
       v[j] = e < N ? row[e] : 0.f;
     }
-    unsigned taken = 0u;  // bit j: expert 32 j + lane is in I_t
-    for (int r = 0; r < k; ++r) {
-      float bv = 0.f;
-      int bi = 0x7fffffff;
+    const int nj = (N + 31) / 32;
+    int ov = 0;
+    for (int sl = 0; sl < k; ++sl) {  // uniform over the warp
+      const int e = cached[t * k + sl];
+      bool ok = e >= 0 && e < N;
+      for (int s2 = 0; ok && s2 < sl; ++s2)
+        if (cached[t * k + s2] == e) ok = false;
+      if (!ok) continue;
+      const float re = row[e];
+      int beat = 0;
 #pragma unroll
       for (int j = 0; j < kPerLane; ++j) {
-        const int e = j * 32 + lane;
-        if (e < N && !((taken >> j) & 1u) && (bi == 0x7fffffff || v[j] > bv)) {
-          bv = v[j];
-          bi = e;
-        }
+        if (j >= nj) break;
+        const int ej = j * 32 + lane;
+        const bool b = ej < N && (v[j] > re || (v[j] == re && ej < e));
+        beat += __popc(__ballot_sync(0xffffffffu, b));
       }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-        if (oi != 0x7fffffff && (bi == 0x7fffffff || ov > bv || (ov == bv && oi < bi))) {
-          bv = ov;
-          bi = oi;
-        }
-      }
-      if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
+      ov += beat < k ? 1 : 0;
     }
-    // Lane s < k checks cached slot s: a valid entry (in range, not repeated in the token) hits
-    // when its owner lane (e & 31) has marked it (bit e >> 5).
-    int e_slot = -1;
-    if (lane < k) {
-      const int e = cached[t * k + lane];
-      bool ok = e >= 0 && e < N;
-      for (int s2 = 0; ok && s2 < lane; ++s2)
-        if (cached[t * k + s2] == e) ok = false;
-      e_slot = ok ? e : -1;
-    }
-    const unsigned owner_mask = __shfl_sync(0xffffffffu, taken, e_slot >= 0 ? (e_slot & 31) : 0);
-    const bool hit = e_slot >= 0 && ((owner_mask >> (e_slot >> 5)) & 1u);
-    const int ov = __popc(__ballot_sync(0xffffffffu, hit));
     if (lane == 0) {
       atomicAdd(&sh_hist[k - ov], 1u);
       atomicAdd(&sh_sum, static_cast<unsigned int>(ov));
@@ -113,9 +100,12 @@ __global__ void __launch_bounds__(256)
 }  // namespace
 
 cudaError_t launch_diagnostics(const float* rho, const int32_t* cached, int64_t T, int N, int k,
-                               int64_t* hist, int64_t* overlap_sum, cudaStream_t st) {
+                               int64_t* hist, int64_t* overlap_sum, int num_sms,
+                               cudaStream_t st) {
   if (T == 0) return cudaSuccess;
-  const unsigned blocks = static_cast<unsigned>((T + kWarps - 1) / kWarps);
+  int64_t want = (T + kWarps - 1) / kWarps;
+  if (want > 2 * static_cast<int64_t>(num_sms)) want = 2 * static_cast<int64_t>(num_sms);
+  const unsigned blocks = static_cast<unsigned>(want);
   return launch_pdl(diagnostics_kernel, dim3(blocks), dim3(kWarps * 32), 0, st, 1, rho, cached,
                     T, N, k, reinterpret_cast<unsigned long long*>(hist),
                     reinterpret_cast<unsigned long long*>(overlap_sum));

@@ -164,7 +164,8 @@ cudaError_t launch_loss_grad_simt(const float* G, const float* h_old, int Tc, in
 
 // ---- diagnostics and feature cache (diagnostics.cu) ---------------------------------------
 cudaError_t launch_diagnostics(const float* rho, const int32_t* cached, int64_t T, int N, int k,
-                               int64_t* hist, int64_t* overlap_sum, cudaStream_t st);
+                               int64_t* hist, int64_t* overlap_sum, int num_sms,
+                               cudaStream_t st);
 cudaError_t launch_feature_cache(const void* h, const float* logits, int64_t T, int64_t Tc,
                                  int d, int N, int esz, int32_t* pos, void* cache_h,
                                  float* cache_p, int num_sms, cudaStream_t st);
