@@ -45,6 +45,8 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU time of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--extras-iters", type=int, default=50,
+                    help="timed calls of each widening row (after 3 untimed)")
     return ap.parse_args()
 
 
@@ -467,7 +469,7 @@ def run_pr2(args, rank, world, local_rank):
                     algorithmic=("flops" if dk["bound"] == "tensor" else "bytes"),
                     per_launch_units=f"{F} token-expert rows x (d={cfg.d}, m={cfg.m})")
 
-    extras = measure_extras(cfg, L, W2, dm, flush, pk)
+    extras = measure_extras(cfg, L, W2, dm, flush, pk, iters=args.extras_iters)
 
     # ---- end to end through the public API with host buffers
     xh = torch.empty(cfg.T, cfg.d, dtype=cfg.torch_dtype, pin_memory=True)
