@@ -7,26 +7,30 @@
 //
 // Persistent kernel: one CTA per SM walks the (M-tile, N-tile) list in M-major order, so the
 // CTAs running at the same time share the weight tiles of the same few experts through L2.
-// Warp 0 issues TMA loads into a STAGES-deep ring of 128-byte-swizzled K-major tiles, warp 1
-// owns TMEM and issues tcgen05.mma (M=128, N=256, K=16) into one of two 256-column fp32
-// accumulators, warps 2..5 drain the other accumulator (one thread per tile row) while the
-// next tile is being multiplied.
+// The A rows (mostly L2 hits: each M-tile is read once per N-tile) and the expert weight tiles
+// (streamed from DRAM) travel in two separate rings of 128-byte-swizzled K-major tiles, each
+// filled by its own TMA warp: warp 0 for A (4 x 16 KB), warp 6 for B (5 x 32 KB), so the
+// long-latency weight stream runs further ahead of the tensor core.  Warp 1 owns TMEM and
+// issues tcgen05.mma (M=128, N=256, K=16) into one of two 256-column fp32 accumulators,
+// warps 2..5 drain the other accumulator (one thread per tile row) while the next tile is being
+// multiplied.
 #include "pr2_device.cuh"
 #include "pr2_internal.h"
 
 namespace pr2 {
 namespace {
 
-constexpr int kThreads = 192;
+constexpr int kThreads = 224;
 constexpr int kBK = 64;
 constexpr int kBN = 256;
-constexpr int kStages = 4;
+constexpr int kStagesA = 4;
+constexpr int kStagesB = 5;
 constexpr int kATile = kTileM * kBK * 2;  // 16 KB
 constexpr int kBTile = kBN * kBK * 2;     // 32 KB
-constexpr int kStageBytes = kATile + kBTile;
+constexpr int kBRing = kStagesA * kATile;  // offset of the B ring
 constexpr int kAccCols = kBN;              // one accumulator
 constexpr uint32_t kTmemCols = 2 * kAccCols;
-constexpr int kBarOffset = kStages * kStageBytes;
+constexpr int kBarOffset = kBRing + kStagesB * kBTile;
 constexpr int kSmemBytes = 1024 + kBarOffset + 256;
 
 template <bool kSwiGLU>
@@ -37,9 +41,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kBarOffset);
-  uint64_t* empty = full + kStages;
-  uint64_t* acc_full = empty + kStages;  // [2]
+  uint64_t* full_a = reinterpret_cast<uint64_t*>(smem + kBarOffset);
+  uint64_t* empty_a = full_a + kStagesA;
+  uint64_t* full_b = empty_a + kStagesA;
+  uint64_t* empty_b = full_b + kStagesB;
+  uint64_t* acc_full = empty_b + kStagesB;  // [2]
   uint64_t* acc_empty = acc_full + 2;    // [2]
   uint64_t* drain = acc_empty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
@@ -52,9 +58,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int KB = g.K / kBK;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+    for (int s = 0; s < kStagesA; ++s) {
+      mbar_init(&full_a[s], 1);
+      mbar_init(&empty_a[s], 1);
+    }
+    for (int s = 0; s < kStagesB; ++s) {
+      mbar_init(&full_b[s], 1);
+      mbar_init(&empty_b[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
@@ -78,8 +88,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_trigger();
   const int num_tiles = (*g.num_tiles) * n_tiles_n;
 
-  if (warp == 0 && lane == 0) {
-    // ---------------- TMA producer ----------------
+  if ((warp == 0 || warp == 6) && lane == 0) {
+    // ---------------- TMA producers: warp 0 the A ring, warp 6 the B ring ----------------
+    const bool is_a = warp == 0;
+    const int nst = is_a ? kStagesA : kStagesB;
+    uint64_t* fullr = is_a ? full_a : full_b;
+    uint64_t* emptyr = is_a ? empty_a : empty_b;
     uint32_t issued = 0, last_par = 0;
     int stage = 0;
     uint32_t phase = 0;
@@ -91,36 +105,40 @@ __global__ void __launch_bounds__(kThreads, 1)
       const TileEntry te = g.tiles[mt];
       const int brow = te.expert * g.b_rows_per_expert + nt * (kSwiGLU ? kBN / 2 : kBN);
       for (int kb = 0; kb < KB; ++kb) {
-        if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, g.status)) {
+        if (!mbar_wait(&emptyr[stage], phase ^ 1u, abort_flag, g.status)) {
           ok = false;
           break;
         }
-        uint8_t* sa = smem + stage * kStageBytes;
-        uint8_t* sb = sa + kATile;
-        mbar_arrive_expect_tx(&full[stage], kStageBytes);
-        tma_load_2d(sa, &tm_a, &full[stage], kb * kBK, te.a_row0);
-        if (kSwiGLU) {
-          tma_load_2d_hint(sb, &tm_b0, &full[stage], kb * kBK, brow, keep);
-          tma_load_2d_hint(sb + kBTile / 2, &tm_b1, &full[stage], kb * kBK, brow, keep);
+        if (is_a) {
+          uint8_t* sa = smem + stage * kATile;
+          mbar_arrive_expect_tx(&fullr[stage], kATile);
+          tma_load_2d(sa, &tm_a, &fullr[stage], kb * kBK, te.a_row0);
         } else {
-          tma_load_2d_hint(sb, &tm_b0, &full[stage], kb * kBK, brow, keep);
+          uint8_t* sb = smem + kBRing + stage * kBTile;
+          mbar_arrive_expect_tx(&fullr[stage], kBTile);
+          if (kSwiGLU) {
+            tma_load_2d_hint(sb, &tm_b0, &fullr[stage], kb * kBK, brow, keep);
+            tma_load_2d_hint(sb + kBTile / 2, &tm_b1, &fullr[stage], kb * kBK, brow, keep);
+          } else {
+            tma_load_2d_hint(sb, &tm_b0, &fullr[stage], kb * kBK, brow, keep);
+          }
         }
         issued |= 1u << stage;
         last_par = (last_par & ~(1u << stage)) | (phase << stage);
-        if (++stage == kStages) {
+        if (++stage == nst) {
           stage = 0;
           phase ^= 1u;
         }
       }
     }
-    for (int s = 0; s < kStages; ++s)
+    for (int s = 0; s < nst; ++s)
       if ((issued >> s) & 1u)
-        mbar_wait_slow(&full[s], (last_par >> s) & 1u, nullptr, nullptr, kDrainLimitNs);
+        mbar_wait_slow(&fullr[s], (last_par >> s) & 1u, nullptr, nullptr, kDrainLimitNs);
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer ----------------
     constexpr uint32_t idesc = umma_idesc_bf16(kTileM, kBN);
-    int stage = 0;
-    uint32_t phase = 0;
+    int sa_i = 0, sb_i = 0;
+    uint32_t pha = 0, phb = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
     bool ok = true;
@@ -129,21 +147,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const uint32_t d_tmem = tmem + acc * kAccCols;
       for (int kb = 0; kb < KB; ++kb) {
-        if (!mbar_wait(&full[stage], phase, abort_flag, g.status)) {
+        if (!mbar_wait(&full_a[sa_i], pha, abort_flag, g.status) ||
+            !mbar_wait(&full_b[sb_i], phb, abort_flag, g.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t sa = smem_u32(smem + stage * kStageBytes);
-        const uint32_t sb = sa + kATile;
+        const uint32_t sa = smem_u32(smem + sa_i * kATile);
+        const uint32_t sb = smem_u32(smem + kBRing + sb_i * kBTile);
 #pragma unroll
         for (int kk = 0; kk < kBK / 16; ++kk)
           umma_bf16(d_tmem, umma_desc_sw128(sa + kk * 32), umma_desc_sw128(sb + kk * 32), idesc,
                     (kb > 0 || kk > 0) ? 1u : 0u);
-        umma_commit(&empty[stage]);
-        if (++stage == kStages) {
-          stage = 0;
-          phase ^= 1u;
+        umma_commit(&empty_a[sa_i]);
+        umma_commit(&empty_b[sb_i]);
+        if (++sa_i == kStagesA) {
+          sa_i = 0;
+          pha ^= 1u;
+        }
+        if (++sb_i == kStagesB) {
+          sb_i = 0;
+          phb ^= 1u;
         }
       }
       if (!ok) break;
@@ -155,7 +179,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     umma_commit(drain);
     mbar_wait_slow(drain, 0, nullptr, nullptr, kDrainLimitNs);
-  } else if (warp >= 2) {
+  } else if (warp >= 2 && warp <= 5) {
     // ---------------- epilogue ----------------
     const int q = warp & 3;
     const int row = q * 32 + lane;
