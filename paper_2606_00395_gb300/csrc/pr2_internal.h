@@ -149,7 +149,7 @@ struct GradArgs {
   float* loss;            // [1]
   int32_t* status;
 };
-constexpr int kLossMaxSplit = 16;
+constexpr int kLossMaxSplit = 8;
 int loss_grad_split(int N, int d, int Tpad, int num_sms);
 cudaError_t launch_loss_grad_tc(const CUtensorMap& tm_gt, const CUtensorMap& tm_h,
                                 const GradArgs& g, cudaStream_t st);

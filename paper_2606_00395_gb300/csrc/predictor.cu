@@ -155,31 +155,30 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// grad = (1/T_c) sum over splits (split order); block 0 also sums the per-token KL in double.
+// grad = (1/T_c) sum over splits (split order, the split loop unrolled against its compile-time
+// maximum so that every partial's load is in flight at once); the last block sums the
+// per-token KL in double in a fixed tree order instead.
 __global__ void __launch_bounds__(256)
     loss_finish_kernel(const float* __restrict__ partial, int split, int64_t n4, float scale,
                        float* __restrict__ grad, const float* __restrict__ kl_tok, int Tc,
                        float* __restrict__ loss) {
   pdl_wait();
   pdl_trigger();
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4;
-       i += stride) {
-    float4 acc = reinterpret_cast<const float4*>(partial)[i];
-    for (int s = 1; s < split; ++s) {
-      const float4 v = reinterpret_cast<const float4*>(partial)[s * n4 + i];
-      acc.x += v.x;
-      acc.y += v.y;
-      acc.z += v.z;
-      acc.w += v.w;
-    }
-    reinterpret_cast<float4*>(grad)[i] =
-        make_float4(acc.x * scale, acc.y * scale, acc.z * scale, acc.w * scale);
-  }
-  if (blockIdx.x == 0) {
+  if (blockIdx.x == gridDim.x - 1) {
     __shared__ double sh[256];
+    double acc[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[j] = 0.0;
+    for (int c0 = 0; c0 < Tc; c0 += 8 * 256) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int c = c0 + j * 256 + static_cast<int>(threadIdx.x);
+        if (c < Tc) acc[j] += static_cast<double>(kl_tok[c]);
+      }
+    }
     double s = 0.0;
-    for (int c = threadIdx.x; c < Tc; c += blockDim.x) s += static_cast<double>(kl_tok[c]);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) s += acc[j];
     sh[threadIdx.x] = s;
     __syncthreads();
     for (int w = 128; w > 0; w >>= 1) {
@@ -187,6 +186,27 @@ __global__ void __launch_bounds__(256)
       __syncthreads();
     }
     if (threadIdx.x == 0) *loss = Tc > 0 ? static_cast<float>(sh[0] / Tc) : 0.f;
+    return;
+  }
+  const int64_t stride = static_cast<int64_t>(gridDim.x - 1) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4;
+       i += stride) {
+    float4 v[kLossMaxSplit];
+#pragma unroll
+    for (int s = 0; s < kLossMaxSplit; ++s)
+      if (s < split) v[s] = reinterpret_cast<const float4*>(partial)[s * n4 + i];
+    float4 acc = v[0];
+#pragma unroll
+    for (int s = 1; s < kLossMaxSplit; ++s) {
+      if (s < split) {
+        acc.x += v[s].x;
+        acc.y += v[s].y;
+        acc.z += v[s].z;
+        acc.w += v[s].w;
+      }
+    }
+    reinterpret_cast<float4*>(grad)[i] =
+        make_float4(acc.x * scale, acc.y * scale, acc.z * scale, acc.w * scale);
   }
 }
 
@@ -327,8 +347,8 @@ cudaError_t launch_loss_finish(const GradArgs& g, cudaStream_t st) {
   // without partials (fp32 path) only the loss is summed
   const int64_t n4 = g.partial != nullptr ? static_cast<int64_t>(g.N) * g.d / 4 : 0;
   int64_t blocks = (n4 + 255) / 256;
-  if (blocks < 1) blocks = 1;
   if (blocks > 1024) blocks = 1024;
+  blocks += 1;  // the last block sums the loss
   const float scale = g.Tc > 0 ? 1.0f / static_cast<float>(g.Tc) : 0.f;
   return launch_pdl(loss_finish_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st, 1,
                     static_cast<const float*>(g.partial), g.split, n4, scale, g.grad, g.kl_tok,
