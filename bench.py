@@ -29,7 +29,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 from paper_2606_00395_gb300 import binding as B  # noqa: E402
-from paper_2606_00395_gb300 import cost, synth  # noqa: E402
+from paper_2606_00395_gb300 import cost, replicas, synth  # noqa: E402
 
 METRIC = "MoE-layer tokens/s (predict-route & replay fwd) on 1 GB300; % of roofline"
 FLUSH_BYTES = 512 << 20
@@ -398,7 +398,8 @@ def run_pr2(args, rank, world, local_rank):
     def el(a, b):
         return a.elapsed_time(b)  # ms
 
-    total_ms = sum(el(e[0], e[6]) for e in evsets)
+    total_ms = replicas.job_time_ms(sum(el(e[0], e[6]) for e in evsets), dist,
+                                    torch.device("cuda", local_rank))
     # per-kernel breakdown: a separate pass with an event at every stage boundary
     n_break = min(args.steps, 200)
     bsets = [make_evs(True) for _ in range(n_break)]
@@ -417,11 +418,7 @@ def run_pr2(args, rank, world, local_rank):
             per["gate_up"].append(el(st[1], st[2]))
             per["down"].append(el(st[2], st[3]))
             per["combine"].append(el(st[3], st[4]))
-    if dist is not None:
-        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-    value = cfg.T * world * args.steps / (total_ms / 1e3)
+    value = replicas.job_throughput(cfg.T * args.steps, world, total_ms)
     mean = {k: statistics.mean(v) for k, v in per.items()}
 
     # ---- per-kernel roofline (algorithmic work / measured duration)
@@ -535,13 +532,9 @@ def run_pr2(args, rank, world, local_rank):
         return start.elapsed_time(end)
 
     run_e2e(max(args.warmup, 2))
-    e2e_total = run_e2e(args.steps)
-    if dist is not None:
-        t = torch.tensor([e2e_total], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_total = float(t.item())
+    e2e_total = replicas.job_time_ms(run_e2e(args.steps), dist, torch.device("cuda", local_rank))
     esz = 2 if cfg.dtype == "bf16" else 4
-    e2e = dict(value=cfg.T * world * args.steps / (e2e_total / 1e3), unit="tokens/s",
+    e2e = dict(value=replicas.job_throughput(cfg.T * args.steps, world, e2e_total), unit="tokens/s",
                h2d_bytes_per_step=cfg.T * cfg.d * esz,
                d2h_bytes_per_step=2 * cfg.T * cfg.d * esz + cfg.T * cfg.k * 4,
                ms_per_step=e2e_total / args.steps,
@@ -606,9 +599,7 @@ def run_reference(args, rank):
 
 def main():
     args = parse()
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    rank, world, local_rank = replicas.rank_env()
     if args.impl == "reference":
         run_reference(args, rank)
         return
