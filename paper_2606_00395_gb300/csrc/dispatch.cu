@@ -102,10 +102,18 @@ __global__ void __launch_bounds__(1024)
   const int g = tid / n_pad, e = tid - g * n_pad;
   const int per = (nblk + G - 1) / G;
   const int b0 = g * per, b1 = min(nblk, b0 + per);
+  // Column slices are read 8 rows at a time with every load in flight (one L2 round trip per
+  // 8 rows instead of a dependent chain).
   int sum = 0;
   if (e < N) {
-#pragma unroll 4
-    for (int b = b0; b < b1; ++b) sum += blk_hist[static_cast<int64_t>(b) * N + e];
+    for (int c0 = b0; c0 < b1; c0 += 8) {
+      int v[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        v[j] = (c0 + j < b1) ? blk_hist[static_cast<int64_t>(c0 + j) * N + e] : 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) sum += v[j];
+    }
   }
   part[tid] = sum;
   __syncthreads();
@@ -138,12 +146,16 @@ __global__ void __launch_bounds__(1024)
   // per-block bases: expert offset + rows of this expert in all earlier blocks
   if (e < N) {
     int run = ex_off[e] + part[g * n_pad + e];
-#pragma unroll 4
-    for (int b = b0; b < b1; ++b) {
-      int32_t* p = blk_hist + static_cast<int64_t>(b) * N + e;
-      const int v = *p;
-      *p = run;
-      run += v;
+    for (int c0 = b0; c0 < b1; c0 += 8) {
+      int v[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        v[j] = (c0 + j < b1) ? blk_hist[static_cast<int64_t>(c0 + j) * N + e] : 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (c0 + j < b1) blk_hist[static_cast<int64_t>(c0 + j) * N + e] = run;
+        run += v[j];
+      }
     }
   }
   // M-tile table: entry i belongs to the expert whose tile range contains i
