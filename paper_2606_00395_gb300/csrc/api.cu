@@ -77,6 +77,7 @@ struct Workspace {
   int32_t* perm;
   int32_t* inv;
   int32_t* num_tiles;
+  unsigned int* sync_ctr;
   TileEntry* tiles;
   TileEntry* stiles1;
   TileEntry* stiles2;
@@ -110,6 +111,7 @@ Workspace carve(const pr2_dims& dm, uint8_t* base) {
   w.perm = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * F));
   w.inv = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * F));
   w.num_tiles = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * 2));
+  w.sync_ctr = reinterpret_cast<unsigned int*>(take(sizeof(unsigned int)));
   w.tiles = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * w.max_tiles));
   w.stiles1 = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * (w.shared_tiles + 1)));
   w.stiles2 = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * (w.shared_tiles + 1)));
@@ -416,7 +418,7 @@ pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* 
   const int es = static_cast<int>(esize(dm));
   DispatchArgs da{idx,       dm.T,       dm.k,      dm.N,    dm.d,   es,     dm.n_shared,
                   w.blk_hist, w.counts,  w.offsets, w.perm,  w.inv,  w.tiles, w.num_tiles,
-                  w.stiles1, w.stiles2,  h,         w.xperm, status};
+                  w.stiles1, w.stiles2,  h,         w.xperm, status, w.sync_ctr};
   if (err == cudaSuccess) err = launch_dispatch(da, num_sms, st);
   mark(events ? events->dispatched : nullptr);
   if (err != cudaSuccess) return PR2_ERR_CUDA;

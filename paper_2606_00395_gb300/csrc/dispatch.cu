@@ -11,9 +11,16 @@
 //               over the 8 warps, then rank = popc(lanes below with the same expert):
 //               perm[offsets[e] + r] = f, inv[f] = its position (-1 for an invalid slot).
 //   4. gather - X[p, :] = h[perm[p] / k, :], 16-byte vectors, one warp per row.
+// Steps 1-3 normally run as one cooperative launch (dispatch_fused_kernel): every block counts
+// its slots, one bounded grid barrier, then each block derives the expert totals, its own
+// per-expert bases and the expert offsets from the whole block histogram (identical in every
+// block), block 0 writes counts, offsets and the tile tables, and every block places its
+// slots.  Shapes whose grid cannot be resident at once use the three kernels above.
 // Combine (the sums of Eqs. pr2_old_output / pr2_output):
 //   out[t, :] = sum_s gates[t,s] * Y[inv[t*k+s], :] + sum_j Ys[j, t, :], fp32 accumulation,
 //   plus, when given, a residual row r[t, :] (the multi-layer loop's h_l; may alias out).
+#include <mutex>
+
 #include "pr2_device.cuh"
 #include "pr2_internal.h"
 
@@ -220,6 +227,226 @@ __global__ void __launch_bounds__(kDispatchChunk)
   }
 }
 
+// Exclusive scan of one int per thread over a 256-thread block (8 warps).
+__device__ __forceinline__ int block256_exclusive_scan(int v, int* sh, int* total) {
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) sh[w] = x;
+  __syncthreads();
+  if (w == 0) {
+    int s = lane < kWarps ? sh[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, s, o);
+      if (lane >= o) s += y;
+    }
+    if (lane < kWarps) sh[lane] = s;
+  }
+  __syncthreads();
+  const int incl = x + (w > 0 ? sh[w - 1] : 0);
+  *total = sh[kWarps - 1];
+  __syncthreads();
+  return incl - v;
+}
+
+// Hist, scan and place in one cooperative launch (N % 4 == 0, N <= 256; grid resident).
+__global__ void __launch_bounds__(kDispatchChunk)
+    dispatch_fused_kernel(const int32_t* __restrict__ idx, int64_t F, int k, int N, int64_t T,
+                          int n_shared, int32_t* blk_hist, int32_t* __restrict__ counts,
+                          int32_t* __restrict__ offsets, int32_t* __restrict__ perm,
+                          int32_t* __restrict__ inv, TileEntry* __restrict__ tiles,
+                          int32_t* __restrict__ num_tiles, TileEntry* __restrict__ stiles1,
+                          TileEntry* __restrict__ stiles2, unsigned int* sync_ctr,
+                          int32_t* status) {
+  extern __shared__ int dsm[];
+  int* wcnt = dsm;                   // [kWarps][N] per-warp counts, then per-warp bases
+  int* tot = wcnt + kWarps * N;      // [N] slots of each expert over all blocks
+  int* pre = tot + N;                // [N] slots of each expert in the blocks before this one
+  int* ex_off = pre + N;             // [N+1]
+  int* ex_tile = ex_off + N + 1;     // [N+1]
+  __shared__ int sh[32];
+  __shared__ int abort_s;
+  pdl_wait();
+  pdl_trigger();
+  const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31;
+  const int nblk = static_cast<int>(gridDim.x), b = static_cast<int>(blockIdx.x);
+  for (int i = tid; i < kWarps * N; i += blockDim.x) wcnt[i] = 0;
+  for (int i = tid; i < N; i += blockDim.x) {
+    tot[i] = 0;
+    pre[i] = 0;
+  }
+  __syncthreads();
+  // ---- 1. this block's slots: validity, per-warp counts, block histogram
+  const int64_t f = static_cast<int64_t>(b) * kDispatchChunk + tid;
+  int e = -1;
+  if (f < F && !slot_valid(idx, f, k, N, &e) && status != nullptr)
+    atomicOr(status, PR2_STATUS_BAD_INDEX);
+  const unsigned same = __match_any_sync(0xffffffffu, e);
+  if (e >= 0 && lane == __ffs(same) - 1) wcnt[w * N + e] = __popc(same);
+  __syncthreads();
+  for (int x = tid; x < N; x += blockDim.x) {
+    int c = 0;
+    for (int ww = 0; ww < kWarps; ++ww) c += wcnt[ww * N + x];
+    blk_hist[static_cast<int64_t>(b) * N + x] = c;
+  }
+  // ---- grid barrier (every block is resident: cooperative launch); bounded
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    atomicAdd(sync_ctr, 1u);
+    const uint64_t t0 = globaltimer_ns();
+    int ok = 1;
+    while (atomicAdd(sync_ctr, 0u) < static_cast<unsigned>(nblk)) {
+      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        ok = 0;
+        if (status != nullptr) atomicOr(status, PR2_STATUS_TIMEOUT);
+        break;
+      }
+    }
+    __threadfence();
+    abort_s = !ok;
+  }
+  __syncthreads();
+  if (abort_s) return;
+  // ---- 2. expert totals and this block's prefix from the whole histogram (int4 columns)
+  const int n4 = N / 4, G = kDispatchChunk / n4;
+  const int q = tid % n4, g = tid / n4;
+  if (g < G) {
+    int4 all = make_int4(0, 0, 0, 0), before = make_int4(0, 0, 0, 0);
+    const int4* col = reinterpret_cast<const int4*>(blk_hist) + q;
+    for (int r0 = g; r0 < nblk; r0 += 8 * G) {
+      int4 v[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int r = r0 + j * G;
+        v[j] = r < nblk ? __ldcg(col + static_cast<int64_t>(r) * n4) : make_int4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int r = r0 + j * G;
+        all.x += v[j].x;
+        all.y += v[j].y;
+        all.z += v[j].z;
+        all.w += v[j].w;
+        if (r < b) {
+          before.x += v[j].x;
+          before.y += v[j].y;
+          before.z += v[j].z;
+          before.w += v[j].w;
+        }
+      }
+    }
+    atomicAdd(&tot[4 * q], all.x);
+    atomicAdd(&tot[4 * q + 1], all.y);
+    atomicAdd(&tot[4 * q + 2], all.z);
+    atomicAdd(&tot[4 * q + 3], all.w);
+    atomicAdd(&pre[4 * q], before.x);
+    atomicAdd(&pre[4 * q + 1], before.y);
+    atomicAdd(&pre[4 * q + 2], before.z);
+    atomicAdd(&pre[4 * q + 3], before.w);
+  }
+  __syncthreads();
+  int all_rows, all_tiles;
+  const int total = tid < N ? tot[tid] : 0;
+  const int off = block256_exclusive_scan(total, sh, &all_rows);
+  const int tstart =
+      block256_exclusive_scan(tid < N ? (total + kTileM - 1) / kTileM : 0, sh, &all_tiles);
+  if (tid < N) {
+    ex_off[tid] = off;
+    ex_tile[tid] = tstart;
+  }
+  if (tid == 0) {
+    ex_off[N] = all_rows;
+    ex_tile[N] = all_tiles;
+  }
+  __syncthreads();
+  if (b == 0) {
+    if (tid < N) {
+      counts[tid] = total;
+      offsets[tid] = off;
+    }
+    if (tid == 0) {
+      offsets[N] = all_rows;
+      num_tiles[0] = all_tiles;
+      num_tiles[1] = n_shared * static_cast<int>((T + kTileM - 1) / kTileM);
+    }
+    for (int i = tid; i < all_tiles; i += blockDim.x) {
+      int lo = 0, hi = N - 1;
+      while (lo < hi) {  // last expert with ex_tile[ex] <= i
+        const int mid = (lo + hi + 1) >> 1;
+        if (ex_tile[mid] <= i) lo = mid; else hi = mid - 1;
+      }
+      const int j = i - ex_tile[lo];
+      const int r0 = ex_off[lo] + j * kTileM;
+      const int left = ex_off[lo + 1] - r0;
+      tiles[i] = TileEntry{lo, r0, left < kTileM ? left : kTileM, r0};
+    }
+    const int mt_T = static_cast<int>((T + kTileM - 1) / kTileM);
+    for (int i = tid; i < n_shared * mt_T; i += blockDim.x) {
+      const int j = i / mt_T, m = i - j * mt_T;
+      const int r0 = m * kTileM;
+      const int rows = (T - r0) < kTileM ? static_cast<int>(T - r0) : kTileM;
+      const int o0 = static_cast<int>(j * T) + r0;
+      stiles1[i] = TileEntry{j, r0, rows, o0};
+      stiles2[i] = TileEntry{j, o0, rows, o0};
+    }
+  }
+  // ---- 3. stable placement: per-warp bases, then ranks within the warp
+  for (int x = tid; x < N; x += blockDim.x) {
+    int run = ex_off[x] + pre[x];
+    for (int ww = 0; ww < kWarps; ++ww) {
+      const int c = wcnt[ww * N + x];
+      wcnt[ww * N + x] = run;
+      run += c;
+    }
+  }
+  __syncthreads();
+  if (f < F) {
+    if (e >= 0) {
+      const int pos = wcnt[w * N + e] + __popc(same & lanemask_lt());
+      perm[pos] = static_cast<int32_t>(f);
+      inv[f] = pos;
+    } else {
+      inv[f] = -1;
+    }
+  }
+}
+
+size_t fused_smem_bytes(int N) { return sizeof(int) * (static_cast<size_t>(kWarps) * N + 4 * N + 2); }
+
+// Whether the fused dispatch can run (shape, and every block resident at once), cached per
+// device and N.
+bool fused_dispatch_ok(int N, int nblk, int num_sms) {
+  if (N % 4 != 0 || N > kDispatchChunk || nblk < 1) return false;
+  struct Entry {
+    int dev, N, blocks_per_sm;
+  };
+  static std::mutex mu;
+  static Entry cache[32];
+  static int used = 0;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  std::lock_guard<std::mutex> lock(mu);
+  int per_sm = -1;
+  for (int i = 0; i < used; ++i)
+    if (cache[i].dev == dev && cache[i].N == N) per_sm = cache[i].blocks_per_sm;
+  if (per_sm < 0) {
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, dispatch_fused_kernel,
+                                                      kDispatchChunk, fused_smem_bytes(N)) !=
+        cudaSuccess) {
+      (void)cudaGetLastError();
+      per_sm = 0;
+    }
+    if (used < 32) cache[used++] = Entry{dev, N, per_sm};
+  }
+  return static_cast<int64_t>(per_sm) * num_sms >= nblk;
+}
+
 // X[p, :] = h[perm[p] / k, :] for p < offsets[N]; row_vec = 16-byte vectors per row.
 __global__ void __launch_bounds__(256)
     gather_kernel(const uint4* __restrict__ h, const int32_t* __restrict__ perm,
@@ -309,19 +536,41 @@ __global__ void __launch_bounds__(256)
 cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st) {
   const int64_t F = a.T * a.k;
   const int nblk = static_cast<int>((F + kDispatchChunk - 1) / kDispatchChunk);
-  if (nblk > 0) {
-    cudaError_t err = launch_pdl(hist_kernel, dim3(nblk), dim3(kDispatchChunk), 0, st, 1,
-                                 a.idx, F, a.k, a.N, a.blk_hist, a.status);
+  cudaError_t err = cudaSuccess;
+  if (nblk > 0 && a.sync_ctr != nullptr && fused_dispatch_ok(a.N, nblk, num_sms)) {
+    err = cudaMemsetAsync(a.sync_ctr, 0, sizeof(unsigned int), st);
     if (err != cudaSuccess) return err;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(nblk);
+    cfg.blockDim = dim3(kDispatchChunk);
+    cfg.dynamicSmemBytes = fused_smem_bytes(a.N);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;  // blocks wait on one another once
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    err = cudaLaunchKernelEx(&cfg, dispatch_fused_kernel, a.idx, F, a.k, a.N, a.T, a.n_shared,
+                             a.blk_hist, a.counts, a.offsets, a.perm, a.inv, a.tiles,
+                             a.num_tiles, a.stiles1, a.stiles2, a.sync_ctr, a.status);
+    if (err != cudaSuccess) return err;
+  } else {
+    if (nblk > 0) {
+      err = launch_pdl(hist_kernel, dim3(nblk), dim3(kDispatchChunk), 0, st, 1, a.idx, F, a.k,
+                       a.N, a.blk_hist, a.status);
+      if (err != cudaSuccess) return err;
+    }
+    err = launch_pdl(scan_kernel, dim3(1), dim3(1024), 0, st, 1, a.blk_hist, nblk, a.N, a.T,
+                     a.n_shared, a.counts, a.offsets, a.tiles, a.num_tiles, a.stiles1,
+                     a.stiles2);
+    if (err != cudaSuccess) return err;
+    if (nblk > 0) {
+      err = launch_pdl(place_kernel, dim3(nblk), dim3(kDispatchChunk), 0, st, 1, a.idx, F, a.k,
+                       a.N, static_cast<const int32_t*>(a.blk_hist), a.perm, a.inv);
+      if (err != cudaSuccess) return err;
+    }
   }
-  cudaError_t err = launch_pdl(scan_kernel, dim3(1), dim3(1024), 0, st, 1, a.blk_hist, nblk, a.N,
-                               a.T, a.n_shared, a.counts, a.offsets, a.tiles, a.num_tiles,
-                               a.stiles1, a.stiles2);
-  if (err != cudaSuccess) return err;
   if (nblk > 0) {
-    err = launch_pdl(place_kernel, dim3(nblk), dim3(kDispatchChunk), 0, st, 1, a.idx, F, a.k,
-                     a.N, static_cast<const int32_t*>(a.blk_hist), a.perm, a.inv);
-    if (err != cudaSuccess) return err;
     const int row_vec = a.d * a.esz / 16;
     int64_t warps_needed = F;
     int64_t blocks = (warps_needed + 7) / 8;

@@ -104,6 +104,7 @@ struct DispatchArgs {
   const void* h;
   void* xperm;           // [T*k, d]
   int32_t* status;
+  unsigned int* sync_ctr;  // grid-barrier counter of the fused dispatch (zeroed per call)
 };
 cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st);
 

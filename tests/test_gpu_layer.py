@@ -17,6 +17,9 @@ pytestmark = pytest.mark.gpu
 SMALL = {
     # fp32 SIMT path, the tiny workload exactly
     "tiny_fp32": synth.CONFIGS["tiny_fp32"],
+    # fp32 with N = 6 experts: dispatch takes its three-kernel path (the fused cooperative
+    # dispatch needs N % 4 == 0)
+    "fp32_n6": synth.LayerConfig("fp32_n6", T=300, d=64, N=6, k=3, m=96, dtype="fp32"),
     # bf16, ~175 rows per expert -> 2 M-tiles per expert, 2 gate/up N-tiles, ragged T
     "bf16_multitile": synth.LayerConfig("bf16_multitile", T=700, d=256, N=16, k=4, m=256),
     # bf16, partial N-tiles in both GEMMs (m = 192 = 128 + 64, d = 320 = 256 + 64), k = 6
