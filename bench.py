@@ -541,7 +541,11 @@ def run_pr2(args, rank, world, local_rank):
                note="copies of neighbouring steps overlap compute on a second stream; "
                     "no L2 flush (1.2 GB of expert weights per step)")
 
-    launches_per_step = 2 + 2 * (7 + (2 if cfg.n_shared else 0))
+    # per layer forward: dispatch (one fused cooperative kernel when N % 4 == 0 and the grid is
+    # resident, as at every bench shape; else hist + scan + place) + gather, the two grouped
+    # GEMMs (+ two for shared experts) and the combine; plus one routing kernel per mode
+    n_dispatch = 2 if cfg.N % 4 == 0 and cfg.N <= 256 else 4
+    launches_per_step = 2 + 2 * (n_dispatch + 3 + (2 if cfg.n_shared else 0))
     line = dict(metric=METRIC, value=value, unit="tokens/s", n_gpus=world, steps=args.steps,
                 warmup=args.warmup, ms_per_step=total_ms / args.steps, higher_is_better=True,
                 scaling="weak", vs_baseline=None, dtype=cfg.dtype, data="synthetic",

@@ -462,7 +462,7 @@ __global__ void __launch_bounds__(256)
     const int t = perm[p] / k;
     const uint4* src = h + static_cast<int64_t>(t) * row_vec;
     uint4* dst = X + static_cast<int64_t>(p) * row_vec;
-#pragma unroll 4
+#pragma unroll 8
     for (int v = lane; v < row_vec; v += 32) dst[v] = __ldg(src + v);
   }
 }
