@@ -277,8 +277,9 @@ def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
         B.check(loop(side), "pr2_rollout_layers (capture)")
     graph_ms = timed(graph.replay, pre=lambda: hd.copy_(h0))
     per_layer = [cost.route_predict_work(Td, cfg.d, cfg.N, cfg.k, cfg.dtype, True),
-                 cost.dispatch_work(Td, cfg.d, cfg.k, cfg.dtype),
-                 cost.expert_gate_up_work(Td * cfg.k, cfg.d, cfg.m, cfg.N, cfg.dtype),
+                 cost.dispatch_work(Td, cfg.d, cfg.k, cfg.dtype, gather=cfg.dtype == "fp32"),
+                 cost.expert_gate_up_work(Td * cfg.k, cfg.d, cfg.m, cfg.N, cfg.dtype,
+                                          a_rows=Td if cfg.dtype == "bf16" else None),
                  cost.expert_down_work(Td * cfg.k, cfg.d, cfg.m, cfg.N, cfg.dtype),
                  cost.combine_work(Td, cfg.d, cfg.k, cfg.n_shared, cfg.dtype)]
     work = cost.KernelWork(Ld * sum(w.bytes for w in per_layer),
@@ -432,8 +433,9 @@ def run_pr2(args, rank, world, local_rank):
     work = {
         "route_predict": cost.route_predict_work(cfg.T, cfg.d, cfg.N, cfg.k, cfg.dtype, True),
         "route_replay": cost.route_replay_work(cfg.T, cfg.d, cfg.N, cfg.k, cfg.dtype, False),
-        "dispatch": cost.dispatch_work(cfg.T, cfg.d, cfg.k, cfg.dtype),
-        "gate_up": cost.expert_gate_up_work(F, cfg.d, cfg.m, hit, cfg.dtype),
+        "dispatch": cost.dispatch_work(cfg.T, cfg.d, cfg.k, cfg.dtype, gather=cfg.dtype == "fp32"),
+        "gate_up": cost.expert_gate_up_work(F, cfg.d, cfg.m, hit, cfg.dtype,
+                                            a_rows=cfg.T if cfg.dtype == "bf16" else None),
         "down": cost.expert_down_work(F, cfg.d, cfg.m, hit, cfg.dtype),
         "combine": cost.combine_work(cfg.T, cfg.d, cfg.k, cfg.n_shared, cfg.dtype),
     }
@@ -542,9 +544,10 @@ def run_pr2(args, rank, world, local_rank):
                     "no L2 flush (1.2 GB of expert weights per step)")
 
     # per layer forward: dispatch (one fused cooperative kernel when N % 4 == 0 and the grid is
-    # resident, as at every bench shape; else hist + scan + place) + gather, the two grouped
-    # GEMMs (+ two for shared experts) and the combine; plus one routing kernel per mode
-    n_dispatch = 2 if cfg.N % 4 == 0 and cfg.N <= 256 else 4
+    # resident, as at every bench shape; else hist + scan + place; + a row gather on the fp32
+    # path only, the bf16 gate/up GEMM gathers its A rows itself), the two grouped GEMMs (+ two
+    # for shared experts) and the combine; plus one routing kernel per mode
+    n_dispatch = (1 if cfg.N % 4 == 0 and cfg.N <= 256 else 3) + (cfg.dtype == "fp32")
     launches_per_step = 2 + 2 * (n_dispatch + 3 + (2 if cfg.n_shared else 0))
     line = dict(metric=METRIC, value=value, unit="tokens/s", n_gpus=world, steps=args.steps,
                 warmup=args.warmup, ms_per_step=total_ms / args.steps, higher_is_better=True,

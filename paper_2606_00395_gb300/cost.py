@@ -59,19 +59,26 @@ def route_replay_work(T: int, d: int, N: int, k: int, dtype: str = "bf16",
     return KernelWork(b, 2 * T * d * N)
 
 
-def dispatch_work(T: int, d: int, k: int, dtype: str = "bf16") -> KernelWork:
-    """Histogram + scan + stable rank + row gather: read idx and h once, write perm, inv and the
-    permuted rows X_perm [T*k, d]."""
+def dispatch_work(T: int, d: int, k: int, dtype: str = "bf16", gather: bool = False) -> KernelWork:
+    """Histogram + scan + stable rank: read idx, write perm and inv.  With `gather` (the fp32
+    path) also read h once and write the permuted rows X_perm [T*k, d]; the bf16 gate/up GEMM
+    reads h through perm itself, so dispatch writes no rows there."""
     e = _esz(dtype)
-    return KernelWork(T * k * 4 + T * d * e + 2 * T * k * 4 + T * k * d * e, 0)
+    b = T * k * 4 + 2 * T * k * 4
+    if gather:
+        b += T * d * e + T * k * d * e
+    return KernelWork(b, 0)
 
 
 def expert_gate_up_work(rows: int, d: int, m: int, experts_hit: int,
-                        dtype: str = "bf16") -> KernelWork:
-    """Grouped [X_e] x [W_gate; W_up]_e^T with the SwiGLU epilogue: read X_perm and the gate/up
-    weights of every expert hit, write H [rows, m]."""
+                        dtype: str = "bf16", a_rows: int | None = None) -> KernelWork:
+    """Grouped [X_e] x [W_gate; W_up]_e^T with the SwiGLU epilogue: read the A rows, the gate/up
+    weights of every expert hit, write H [rows, m].  `a_rows` is the number of distinct A rows
+    that must cross HBM: the T tokens of h when the GEMM gathers them (each token feeds k
+    rows), `rows` when it reads a permuted copy."""
     e = _esz(dtype)
-    return KernelWork(rows * d * e + experts_hit * 2 * m * d * e + rows * m * e,
+    a = rows if a_rows is None else a_rows
+    return KernelWork(a * d * e + experts_hit * 2 * m * d * e + rows * m * e,
                       2 * rows * d * 2 * m)
 
 

@@ -115,7 +115,8 @@ Workspace carve(const pr2_dims& dm, uint8_t* base) {
   w.tiles = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * w.max_tiles));
   w.stiles1 = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * (w.shared_tiles + 1)));
   w.stiles2 = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * (w.shared_tiles + 1)));
-  w.xperm = take(es * F * dm.d);
+  // permuted copy of h: only the fp32 path reads it; the bf16 gate/up GEMM gathers from h
+  w.xperm = dm.dtype == PR2_FP32 ? take(es * F * dm.d) : nullptr;
   w.hbuf = take(es * F * dm.m);
   w.ybuf = take(es * F * dm.d);
   w.hs = take(es * dm.n_shared * dm.T * dm.m);
@@ -419,18 +420,23 @@ pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* 
   DispatchArgs da{idx,       dm.T,       dm.k,      dm.N,    dm.d,   es,     dm.n_shared,
                   w.blk_hist, w.counts,  w.offsets, w.perm,  w.inv,  w.tiles, w.num_tiles,
                   w.stiles1, w.stiles2,  h,         w.xperm, status, w.sync_ctr};
+  // (w.xperm is nullptr on the bf16 path: dispatch then launches no gather)
   if (err == cudaSuccess) err = launch_dispatch(da, num_sms, st);
   mark(events ? events->dispatched : nullptr);
   if (err != cudaSuccess) return PR2_ERR_CUDA;
 
   const int64_t F = dm.T * dm.k;
-  GemmArgs g1{w.tiles, w.num_tiles, w.max_tiles, dm.d, dm.m, dm.m, w.hbuf, status};
-  GemmArgs g2{w.tiles, w.num_tiles, w.max_tiles, dm.m, dm.d, dm.d, w.ybuf, status};
-  GemmArgs s1{w.stiles1, w.num_tiles + 1, w.shared_tiles, dm.d, dm.m, dm.m, w.hs, status};
-  GemmArgs s2{w.stiles2, w.num_tiles + 1, w.shared_tiles, dm.m, dm.d, dm.d, w.ys, status};
+  GemmArgs g1{w.tiles, w.num_tiles, w.max_tiles, dm.d, dm.m, dm.m, w.hbuf, status,
+              h, w.perm, dm.k};  // gathered A (bf16); the fp32 GEMM reads w.xperm
+  GemmArgs g2{w.tiles, w.num_tiles, w.max_tiles, dm.m, dm.d, dm.d, w.ybuf, status,
+              nullptr, nullptr, 0};
+  GemmArgs s1{w.stiles1, w.num_tiles + 1, w.shared_tiles, dm.d, dm.m, dm.m, w.hs, status,
+              nullptr, nullptr, 0};
+  GemmArgs s2{w.stiles2, w.num_tiles + 1, w.shared_tiles, dm.m, dm.d, dm.d, w.ys, status,
+              nullptr, nullptr, 0};
   if (dm.dtype == PR2_BF16) {
     CUtensorMap a1, b1g, b1u, a2, b2, sa1, sb1g, sb1u, sa2, sb2;
-    bool ok = make_tmap_bf16(&a1, w.xperm, dm.d, F, 64, kTileM) &&
+    bool ok = make_tmap_bf16(&a1, h, dm.d, dm.T, 64, kTileM) &&  // unused: A is gathered
               make_tmap_bf16(&b1g, W_gate, dm.d, (uint64_t)dm.N * dm.m, 64, 128) &&
               make_tmap_bf16(&b1u, W_up, dm.d, (uint64_t)dm.N * dm.m, 64, 128) &&
               make_tmap_bf16(&a2, w.hbuf, dm.m, F, 64, kTileM) &&
@@ -443,13 +449,13 @@ pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* 
            make_tmap_bf16(&sb2, Ws_down, dm.m, (uint64_t)dm.n_shared * dm.d, 64, 256);
     }
     if (!ok) return PR2_ERR_CUDA;
-    err = launch_expert_tc(true, a1, b1g, b1u, g1, num_sms, st);
+    err = launch_expert_tc(true, true, a1, b1g, b1u, g1, num_sms, st);
     if (err == cudaSuccess && dm.n_shared > 0)
-      err = launch_expert_tc(true, sa1, sb1g, sb1u, s1, num_sms, st);
+      err = launch_expert_tc(true, false, sa1, sb1g, sb1u, s1, num_sms, st);
     mark(events ? events->gate_up_done : nullptr);
-    if (err == cudaSuccess) err = launch_expert_tc(false, a2, b2, b2, g2, num_sms, st);
+    if (err == cudaSuccess) err = launch_expert_tc(false, false, a2, b2, b2, g2, num_sms, st);
     if (err == cudaSuccess && dm.n_shared > 0)
-      err = launch_expert_tc(false, sa2, sb2, sb2, s2, num_sms, st);
+      err = launch_expert_tc(false, false, sa2, sb2, sb2, s2, num_sms, st);
     mark(events ? events->down_done : nullptr);
   } else {
     err = launch_expert_simt(true, static_cast<const float*>(w.xperm),

@@ -570,7 +570,7 @@ cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st)
       if (err != cudaSuccess) return err;
     }
   }
-  if (nblk > 0) {
+  if (nblk > 0 && a.xperm != nullptr) {
     const int row_vec = a.d * a.esz / 16;
     int64_t warps_needed = F;
     int64_t blocks = (warps_needed + 7) / 8;

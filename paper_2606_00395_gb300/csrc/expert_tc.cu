@@ -4,36 +4,98 @@
 // grouped by expert:
 //   gate/up GEMM:  H[r, :] = silu(X[r] Wg_e^T) * (X[r] Wu_e^T)     (K = d, 128 H columns / tile)
 //   down GEMM:     Y[r, :] = H[r] Wd_e^T                           (K = m, 256 Y columns / tile)
+// where X[r] = h[perm[r] / k] is the token that dispatch placed at row r.
 //
 // Persistent kernel: one CTA per SM walks the (M-tile, N-tile) list in M-major order, so the
 // CTAs running at the same time share the weight tiles of the same few experts through L2.
-// The A rows (mostly L2 hits: each M-tile is read once per N-tile) and the expert weight tiles
-// (streamed from DRAM) travel in two separate rings of 128-byte-swizzled K-major tiles, each
-// filled by its own TMA warp: warp 0 for A (4 x 16 KB), warp 6 for B (5 x 32 KB), so the
-// long-latency weight stream runs further ahead of the tensor core.  Warp 1 owns TMEM and
-// issues tcgen05.mma (M=128, N=256, K=16) into one of two 256-column fp32 accumulators,
-// warps 2..5 drain the other accumulator (one thread per tile row) while the next tile is being
-// multiplied.
+// The A rows and the expert weight tiles (streamed from DRAM) travel in two separate rings of
+// 128-byte-swizzled K-major tiles (A 4 x 16 KB, B 5 x 32 KB), so the long-latency weight stream
+// runs further ahead of the tensor core.  Warp roles:
+//   warps 0-3  A producers.  Gate/up GEMM of the routed experts: all 128 threads gather the
+//              tile's rows straight from h with 16-byte cp.async (each thread owns 8 rows and
+//              one 16-byte column chunk, written to its swizzled position), so neither a
+//              permuted copy of h nor a gather launch exists; h (T x d) stays in L2.  Other
+//              GEMMs: one thread issues TMA loads of the A tile.
+//   warp 4     TMEM owner and tcgen05.mma issuer (M=128, N=256, K=16) into one of two
+//              256-column fp32 accumulators.
+//   warp 5     TMA producer of the weight ring.
+//   warps 6-9  epilogue: drain the other accumulator (one thread per tile row) while the next
+//              tile is being multiplied.
 #include "pr2_device.cuh"
 #include "pr2_internal.h"
 
 namespace pr2 {
 namespace {
 
-constexpr int kThreads = 224;
+constexpr int kThreads = 320;
+constexpr int kWarpMma = 4;
+constexpr int kWarpB = 5;
 constexpr int kBK = 64;
 constexpr int kBN = 256;
 constexpr int kStagesA = 4;
 constexpr int kStagesB = 5;
-constexpr int kATile = kTileM * kBK * 2;  // 16 KB
-constexpr int kBTile = kBN * kBK * 2;     // 32 KB
-constexpr int kBRing = kStagesA * kATile;  // offset of the B ring
-constexpr int kAccCols = kBN;              // one accumulator
+constexpr int kGatherThreads = 128;         // warps 0-3
+constexpr int kATile = kTileM * kBK * 2;    // 16 KB
+constexpr int kBTile = kBN * kBK * 2;       // 32 KB
+constexpr int kBRing = kStagesA * kATile;   // offset of the B ring
+constexpr int kAccCols = kBN;               // one accumulator
 constexpr uint32_t kTmemCols = 2 * kAccCols;
 constexpr int kBarOffset = kBRing + kStagesB * kBTile;
 constexpr int kSmemBytes = 1024 + kBarOffset + 256;
 
-template <bool kSwiGLU>
+// A producer of the gathered gate/up GEMM: thread `tid` of warps 0-3 copies, for every K block,
+// the 16-byte chunk `c = tid % 8` of tile rows r = tid / 8 + 16 i (i = 0..7).  In the 128-byte
+// swizzled K-major tile, chunk c of row r sits at r * 128 + ((c ^ (r % 8)) * 16), and r % 8 is
+// the same for all eight rows of a thread.  After its eight copies of a stage the thread
+// registers an arrival on that stage's full barrier (count 128) that fires when they have
+// landed; the MMA thread, after acquiring the barrier, fences the stage into the async proxy.
+__device__ __forceinline__ void gather_a_producer(const GemmArgs& g, uint8_t* smem,
+                                                  uint64_t* full_a, uint64_t* empty_a,
+                                                  volatile int* abort_flag, int n_tiles_n,
+                                                  int num_tiles, int KB) {
+  const int tid = threadIdx.x;
+  const int c = tid & 7;
+  const int r0 = tid >> 3;
+  const uint32_t soff = static_cast<uint32_t>(r0 * 128 + ((c ^ (r0 & 7)) << 4));
+  const __nv_bfloat16* h = static_cast<const __nv_bfloat16*>(g.a_src);
+  const int64_t ld = g.K;
+  const uint64_t keep = l2_policy_evict_last();  // h: every token row is read k times
+  int stage = 0;
+  uint32_t phase = 0;
+  bool ok = true;
+  for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+    const TileEntry te = g.tiles[tile / n_tiles_n];
+    const __nv_bfloat16* src[8];
+    uint32_t nbytes[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int row = r0 + 16 * i;
+      const bool live = row < te.rows;
+      const int64_t t = live ? g.perm[te.a_row0 + row] / g.k : 0;
+      src[i] = h + t * ld + c * 8;  // padding rows: zero-filled, nothing read
+      nbytes[i] = live ? 16u : 0u;
+    }
+    for (int kb = 0; kb < KB; ++kb) {
+      if (!mbar_wait(&empty_a[stage], phase ^ 1u, abort_flag, g.status)) {
+        ok = false;
+        break;
+      }
+      const uint32_t dst = smem_u32(smem + stage * kATile) + soff;
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        cp_async_16_hint(dst + i * 2048, src[i] + kb * kBK, nbytes[i], keep);
+      cp_async_arrive_noinc(&full_a[stage]);
+      if (++stage == kStagesA) {
+        stage = 0;
+        phase ^= 1u;
+      }
+    }
+  }
+  cp_async_commit();
+  cp_async_wait<0>();  // nothing may still be writing shared memory when the CTA leaves
+}
+
+template <bool kSwiGLU, bool kGatherA>
 __global__ void __launch_bounds__(kThreads, 1)
     expert_tc_kernel(const __grid_constant__ CUtensorMap tm_a,
                      const __grid_constant__ CUtensorMap tm_b0,
@@ -59,7 +121,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStagesA; ++s) {
-      mbar_init(&full_a[s], 1);
+      mbar_init(&full_a[s], kGatherA ? kGatherThreads : 1);
       mbar_init(&empty_a[s], 1);
     }
     for (int s = 0; s < kStagesB; ++s) {
@@ -73,11 +135,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
-    tma_prefetch_desc(&tm_a);
+    if (!kGatherA) tma_prefetch_desc(&tm_a);
     tma_prefetch_desc(&tm_b0);
     if (kSwiGLU) tma_prefetch_desc(&tm_b1);
   }
-  if (warp == 1) {
+  if (warp == kWarpMma) {
     tmem_alloc(tmem_slot, kTmemCols);
     tc_fence_before();
   }
@@ -88,8 +150,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_trigger();
   const int num_tiles = (*g.num_tiles) * n_tiles_n;
 
-  if ((warp == 0 || warp == 6) && lane == 0) {
-    // ---------------- TMA producers: warp 0 the A ring, warp 6 the B ring ----------------
+  if (kGatherA && warp < 4) {
+    gather_a_producer(g, smem, full_a, empty_a, abort_flag, n_tiles_n, num_tiles, KB);
+  } else if ((warp == 0 || warp == kWarpB) && lane == 0) {
+    // ---------------- TMA producers: warp 0 the A ring, warp 5 the B ring ----------------
     const bool is_a = warp == 0;
     const int nst = is_a ? kStagesA : kStagesB;
     uint64_t* fullr = is_a ? full_a : full_b;
@@ -97,13 +161,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t issued = 0, last_par = 0;
     int stage = 0;
     uint32_t phase = 0;
-    const uint64_t keep = l2_policy_evict_last();  // expert weights: reused by every M-tile
+    // Expert weights are reused by the M-tiles of their expert, which run at about the same
+    // time: evict_last keeps them for the down GEMM; the gathered GEMM keeps h instead.
+    const uint64_t keep = l2_policy_evict_last();
     bool ok = true;
     for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
       const int mt = tile / n_tiles_n;
       const int nt = tile - mt * n_tiles_n;
       const TileEntry te = g.tiles[mt];
-      const int brow = te.expert * g.b_rows_per_expert + nt * (kSwiGLU ? kBN / 2 : kBN);
+      const int brow = te.expert * g.b_rows_per_expert + nt * kColsPerTile;
       for (int kb = 0; kb < KB; ++kb) {
         if (!mbar_wait(&emptyr[stage], phase ^ 1u, abort_flag, g.status)) {
           ok = false;
@@ -116,7 +182,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         } else {
           uint8_t* sb = smem + kBRing + stage * kBTile;
           mbar_arrive_expect_tx(&fullr[stage], kBTile);
-          if (kSwiGLU) {
+          if (kGatherA) {
+            tma_load_2d(sb, &tm_b0, &fullr[stage], kb * kBK, brow);
+            tma_load_2d(sb + kBTile / 2, &tm_b1, &fullr[stage], kb * kBK, brow);
+          } else if (kSwiGLU) {
             tma_load_2d_hint(sb, &tm_b0, &fullr[stage], kb * kBK, brow, keep);
             tma_load_2d_hint(sb + kBTile / 2, &tm_b1, &fullr[stage], kb * kBK, brow, keep);
           } else {
@@ -134,7 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = 0; s < nst; ++s)
       if ((issued >> s) & 1u)
         mbar_wait_slow(&fullr[s], (last_par >> s) & 1u, nullptr, nullptr, kDrainLimitNs);
-  } else if (warp == 1 && lane == 0) {
+  } else if (warp == kWarpMma && lane == 0) {
     // ---------------- MMA issuer ----------------
     constexpr uint32_t idesc = umma_idesc_bf16(kTileM, kBN);
     int sa_i = 0, sb_i = 0;
@@ -152,6 +221,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = false;
           break;
         }
+        if (kGatherA) fence_proxy_async_smem();  // rows written by cp.async (generic proxy)
         tc_fence_after();
         const uint32_t sa = smem_u32(smem + sa_i * kATile);
         const uint32_t sb = smem_u32(smem + kBRing + sb_i * kBTile);
@@ -179,8 +249,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     umma_commit(drain);
     mbar_wait_slow(drain, 0, nullptr, nullptr, kDrainLimitNs);
-  } else if (warp >= 2 && warp <= 5) {
-    // ---------------- epilogue ----------------
+  } else if (warp >= 6) {
+    // ---------------- epilogue (warp w reads TMEM lanes 32 (w % 4) .. +31) ----------------
     const int q = warp & 3;
     const int row = q * 32 + lane;
     int acc = 0;
@@ -247,7 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   __syncthreads();
-  if (warp == 1) {
+  if (warp == kWarpMma) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
@@ -255,14 +325,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-cudaError_t launch_expert_tc(bool swiglu, const CUtensorMap& tm_a, const CUtensorMap& tm_b0,
-                             const CUtensorMap& tm_b1, const GemmArgs& g, int num_sms,
-                             cudaStream_t st) {
+cudaError_t launch_expert_tc(bool swiglu, bool gather_a, const CUtensorMap& tm_a,
+                             const CUtensorMap& tm_b0, const CUtensorMap& tm_b1,
+                             const GemmArgs& g, int num_sms, cudaStream_t st) {
   if (g.max_tiles <= 0) return cudaSuccess;
+  if (gather_a && (!swiglu || g.a_src == nullptr || g.perm == nullptr || g.k <= 0))
+    return cudaErrorInvalidValue;
   const int cols = swiglu ? kBN / 2 : kBN;
   const int64_t bound = static_cast<int64_t>(g.max_tiles) * ((g.n_out + cols - 1) / cols);
   const int grid = static_cast<int>(bound < num_sms ? bound : num_sms);
-  auto* kernel = swiglu ? expert_tc_kernel<true> : expert_tc_kernel<false>;
+  auto* kernel = gather_a ? expert_tc_kernel<true, true>
+                          : (swiglu ? expert_tc_kernel<true, false> : expert_tc_kernel<false, false>);
   const cudaError_t err =
       cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   if (err != cudaSuccess) return err;

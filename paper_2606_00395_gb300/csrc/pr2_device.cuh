@@ -126,6 +126,42 @@ __device__ __forceinline__ void tma_load_2d_hint(void* smem_dst, const void* tma
       : "memory");
 }
 
+// ------------------------------------------------------------------------------------------
+// Per-thread 16-byte asynchronous copies global -> shared (cp.async), for row gathers that a
+// tensor map cannot express.  `src_bytes` = 0 fills the 16 bytes with zeros (nothing is read).
+// cp_async_arrive_noinc makes an mbarrier arrival fire once all of the thread's earlier
+// cp.async copies have landed (the barrier's count includes these arrivals).  The data is
+// written through the generic proxy: the thread that acquires the barrier executes
+// fence.proxy.async before a tcgen05.mma (async proxy) reads it.
+// ------------------------------------------------------------------------------------------
+__device__ __forceinline__ void cp_async_16(uint32_t smem_dst, const void* src,
+                                            uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_dst), "l"(src),
+               "r"(src_bytes)
+               : "memory");
+}
+// Same with an L2 eviction-priority hint (a createpolicy value).
+__device__ __forceinline__ void cp_async_16_hint(uint32_t smem_dst, const void* src,
+                                                 uint32_t src_bytes, uint64_t policy) {
+  asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2, %3;" ::"r"(smem_dst),
+               "l"(src), "r"(src_bytes), "l"(policy)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_arrive_noinc(uint64_t* bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int kPending>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(kPending) : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 __device__ __forceinline__ uint64_t l2_policy_evict_last() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));

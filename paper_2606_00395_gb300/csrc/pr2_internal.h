@@ -102,7 +102,7 @@ struct DispatchArgs {
   TileEntry* stiles1;    // [n_shared * ceil(T/128)] gate/up GEMM of the shared experts
   TileEntry* stiles2;    // same, down GEMM
   const void* h;
-  void* xperm;           // [T*k, d]
+  void* xperm;           // [T*k, d] permuted copy of h (fp32 path); nullptr: no gather launch
   int32_t* status;
   unsigned int* sync_ctr;  // grid-barrier counter of the fused dispatch (zeroed per call)
 };
@@ -130,11 +130,18 @@ struct GemmArgs {
   int b_rows_per_expert;     // rows of one expert's weight matrix (m for gate/up, d for down)
   void* out;                 // [rows, n_out]
   int32_t* status;
+  // Gathered A (gate/up GEMM of the routed experts): row r of a tile is token perm[r] / k of
+  // `a_src` [T, K] instead of row r of a permuted copy.  Unused when the A operand comes from
+  // the tensor map.
+  const void* a_src;
+  const int32_t* perm;
+  int k;
 };
 // swiglu: out = silu(A Wg^T) * (A Wu^T) (tm_b0 = gate, tm_b1 = up); else out = A Wb^T.
-cudaError_t launch_expert_tc(bool swiglu, const CUtensorMap& tm_a, const CUtensorMap& tm_b0,
-                             const CUtensorMap& tm_b1, const GemmArgs& g, int num_sms,
-                             cudaStream_t st);
+// gather_a: A rows are read from g.a_src through g.perm (tm_a unused); else from tm_a.
+cudaError_t launch_expert_tc(bool swiglu, bool gather_a, const CUtensorMap& tm_a,
+                             const CUtensorMap& tm_b0, const CUtensorMap& tm_b1,
+                             const GemmArgs& g, int num_sms, cudaStream_t st);
 cudaError_t launch_expert_simt(bool swiglu, const float* A, const float* Wb0, const float* Wb1,
                                const GemmArgs& g, cudaStream_t st);
 

@@ -33,9 +33,12 @@ def test_workspace_bytes_grow_with_the_layer(lib):
     big = B.pr2_moe_workspace_bytes(B.dims(4096, 2048, 128, 8, 768))
     shared = B.pr2_moe_workspace_bytes(B.dims(4096, 2048, 128, 8, 768, n_shared=1))
     assert 0 < small < big < shared
-    # dominated by the permuted rows, the expert hidden activations and the expert outputs
+    # bf16: dominated by the expert hidden activations and the expert outputs (the gate/up GEMM
+    # gathers its rows from h, so there is no permuted copy); fp32 adds the permuted rows
     F = 4096 * 8
-    assert big >= 2 * F * (2048 + 768 + 2048)
+    assert 2 * F * (768 + 2048) <= big < 2 * F * (768 + 2048) + 2 * F * 2048
+    big32 = B.pr2_moe_workspace_bytes(B.dims(4096, 2048, 128, 8, 768, dtype="fp32"))
+    assert big32 >= 4 * F * (2048 + 768 + 2048)
 
 
 @pytest.mark.parametrize("bad", [
