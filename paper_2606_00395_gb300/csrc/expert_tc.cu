@@ -21,6 +21,10 @@
 //   warp 5     TMA producer of the weight ring.
 //   warps 6-9  epilogue: drain the other accumulator (one thread per tile row) while the next
 //              tile is being multiplied.
+// Each tcgen05.commit costs the tensor pipe about 25 ns (a third of one MMA), so the MMA thread
+// commits once per K block, to the weight ring's empty barrier.  That completion also frees the
+// A stage the K block used: the A producers wait on the weight ring's barrier of the K block
+// kStagesA earlier instead of on a barrier of their own.
 #include "pr2_device.cuh"
 #include "pr2_internal.h"
 
@@ -42,6 +46,28 @@ constexpr int kAccCols = kBN;               // one accumulator
 constexpr uint32_t kTmemCols = 2 * kAccCols;
 constexpr int kBarOffset = kBRing + kStagesB * kBTile;
 constexpr int kSmemBytes = 1024 + kBarOffset + 256;
+// The A producer's wait on empty_b relies on that barrier never being two phases ahead of it.
+static_assert(kStagesA <= kStagesB, "the A ring may not be deeper than the weight ring");
+
+// Where the A producer learns that an A stage is free: K block n reuses the A stage of K block
+// j = n - kStagesA, whose MMAs completed phase j / kStagesB of empty_b[j % kStagesB].
+struct ReleaseCursor {
+  int n = 0;          // K blocks issued so far
+  int slot = 0;       // empty_b slot of K block n - kStagesA
+  uint32_t par = 0;   // its phase parity
+  __device__ __forceinline__ bool wait(uint64_t* empty_b, volatile int* abort_flag,
+                                       int32_t* status) {
+    if (n < kStagesA) return true;
+    return mbar_wait(&empty_b[slot], par, abort_flag, status);
+  }
+  __device__ __forceinline__ void advance() {
+    if (n++ < kStagesA) return;
+    if (++slot == kStagesB) {
+      slot = 0;
+      par ^= 1u;
+    }
+  }
+};
 
 // A producer of the gathered gate/up GEMM: thread `tid` of warps 0-3 copies, for every K block,
 // the 16-byte chunk `c = tid % 8` of tile rows r = tid / 8 + 16 i (i = 0..7).  In the 128-byte
@@ -50,7 +76,7 @@ constexpr int kSmemBytes = 1024 + kBarOffset + 256;
 // registers an arrival on that stage's full barrier (count 128) that fires when they have
 // landed; the MMA thread, after acquiring the barrier, fences the stage into the async proxy.
 __device__ __forceinline__ void gather_a_producer(const GemmArgs& g, uint8_t* smem,
-                                                  uint64_t* full_a, uint64_t* empty_a,
+                                                  uint64_t* full_a, uint64_t* empty_b,
                                                   volatile int* abort_flag, int n_tiles_n,
                                                   int num_tiles, int KB) {
   const int tid = threadIdx.x;
@@ -61,7 +87,7 @@ __device__ __forceinline__ void gather_a_producer(const GemmArgs& g, uint8_t* sm
   const int64_t ld = g.K;
   const uint64_t keep = l2_policy_evict_last();  // h: every token row is read k times
   int stage = 0;
-  uint32_t phase = 0;
+  ReleaseCursor rel;
   bool ok = true;
   for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
     const TileEntry te = g.tiles[tile / n_tiles_n];
@@ -76,19 +102,17 @@ __device__ __forceinline__ void gather_a_producer(const GemmArgs& g, uint8_t* sm
       nbytes[i] = live ? 16u : 0u;
     }
     for (int kb = 0; kb < KB; ++kb) {
-      if (!mbar_wait(&empty_a[stage], phase ^ 1u, abort_flag, g.status)) {
+      if (!rel.wait(empty_b, abort_flag, g.status)) {
         ok = false;
         break;
       }
+      rel.advance();
       const uint32_t dst = smem_u32(smem + stage * kATile) + soff;
 #pragma unroll
       for (int i = 0; i < 8; ++i)
         cp_async_16_hint(dst + i * 2048, src[i] + kb * kBK, nbytes[i], keep);
       cp_async_arrive_noinc(&full_a[stage]);
-      if (++stage == kStagesA) {
-        stage = 0;
-        phase ^= 1u;
-      }
+      if (++stage == kStagesA) stage = 0;
     }
   }
   cp_async_commit();
@@ -104,8 +128,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* full_a = reinterpret_cast<uint64_t*>(smem + kBarOffset);
-  uint64_t* empty_a = full_a + kStagesA;
-  uint64_t* full_b = empty_a + kStagesA;
+  uint64_t* full_b = full_a + kStagesA;
   uint64_t* empty_b = full_b + kStagesB;
   uint64_t* acc_full = empty_b + kStagesB;  // [2]
   uint64_t* acc_empty = acc_full + 2;    // [2]
@@ -120,10 +143,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int KB = g.K / kBK;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStagesA; ++s) {
-      mbar_init(&full_a[s], kGatherA ? kGatherThreads : 1);
-      mbar_init(&empty_a[s], 1);
-    }
+    for (int s = 0; s < kStagesA; ++s) mbar_init(&full_a[s], kGatherA ? kGatherThreads : 1);
     for (int s = 0; s < kStagesB; ++s) {
       mbar_init(&full_b[s], 1);
       mbar_init(&empty_b[s], 1);
@@ -151,19 +171,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int num_tiles = (*g.num_tiles) * n_tiles_n;
 
   if (kGatherA && warp < 4) {
-    gather_a_producer(g, smem, full_a, empty_a, abort_flag, n_tiles_n, num_tiles, KB);
+    gather_a_producer(g, smem, full_a, empty_b, abort_flag, n_tiles_n, num_tiles, KB);
   } else if ((warp == 0 || warp == kWarpB) && lane == 0) {
     // ---------------- TMA producers: warp 0 the A ring, warp 5 the B ring ----------------
     const bool is_a = warp == 0;
     const int nst = is_a ? kStagesA : kStagesB;
     uint64_t* fullr = is_a ? full_a : full_b;
-    uint64_t* emptyr = is_a ? empty_a : empty_b;
     uint32_t issued = 0, last_par = 0;
     int stage = 0;
     uint32_t phase = 0;
-    // Expert weights are reused by the M-tiles of their expert, which run at about the same
-    // time: evict_last keeps them for the down GEMM; the gathered GEMM keeps h instead.
-    const uint64_t keep = l2_policy_evict_last();
+    ReleaseCursor rel;  // A ring: stage release through the weight ring's barriers
+    // Expert weights are reused only by the M-tiles of their expert, which run at about the
+    // same time, so they take the normal L2 policy (an evict_last hint on them pushes out h,
+    // H and Y, which later tiles and kernels read again).
     bool ok = true;
     for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
       const int mt = tile / n_tiles_n;
@@ -171,26 +191,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       const TileEntry te = g.tiles[mt];
       const int brow = te.expert * g.b_rows_per_expert + nt * kColsPerTile;
       for (int kb = 0; kb < KB; ++kb) {
-        if (!mbar_wait(&emptyr[stage], phase ^ 1u, abort_flag, g.status)) {
+        const bool free = is_a ? rel.wait(empty_b, abort_flag, g.status)
+                               : mbar_wait(&empty_b[stage], phase ^ 1u, abort_flag, g.status);
+        if (!free) {
           ok = false;
           break;
         }
         if (is_a) {
+          rel.advance();
           uint8_t* sa = smem + stage * kATile;
           mbar_arrive_expect_tx(&fullr[stage], kATile);
           tma_load_2d(sa, &tm_a, &fullr[stage], kb * kBK, te.a_row0);
         } else {
           uint8_t* sb = smem + kBRing + stage * kBTile;
           mbar_arrive_expect_tx(&fullr[stage], kBTile);
-          if (kGatherA) {
-            tma_load_2d(sb, &tm_b0, &fullr[stage], kb * kBK, brow);
-            tma_load_2d(sb + kBTile / 2, &tm_b1, &fullr[stage], kb * kBK, brow);
-          } else if (kSwiGLU) {
-            tma_load_2d_hint(sb, &tm_b0, &fullr[stage], kb * kBK, brow, keep);
-            tma_load_2d_hint(sb + kBTile / 2, &tm_b1, &fullr[stage], kb * kBK, brow, keep);
-          } else {
-            tma_load_2d_hint(sb, &tm_b0, &fullr[stage], kb * kBK, brow, keep);
-          }
+          tma_load_2d(sb, &tm_b0, &fullr[stage], kb * kBK, brow);
+          if (kSwiGLU) tma_load_2d(sb + kBTile / 2, &tm_b1, &fullr[stage], kb * kBK, brow);
         }
         issued |= 1u << stage;
         last_par = (last_par & ~(1u << stage)) | (phase << stage);
@@ -229,8 +245,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kk = 0; kk < kBK / 16; ++kk)
           umma_bf16(d_tmem, umma_desc_sw128(sa + kk * 32), umma_desc_sw128(sb + kk * 32), idesc,
                     (kb > 0 || kk > 0) ? 1u : 0u);
-        umma_commit(&empty_a[sa_i]);
-        umma_commit(&empty_b[sb_i]);
+        umma_commit(&empty_b[sb_i]);  // frees this K block's weight stage and A stage
         if (++sa_i == kStagesA) {
           sa_i = 0;
           pha ^= 1u;
