@@ -477,7 +477,7 @@ pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* 
   if (err != cudaSuccess) return PR2_ERR_CUDA;
 
   CombineArgs ca{w.ybuf, dm.n_shared > 0 ? w.ys : nullptr, w.inv, gates, dm.T, dm.k, dm.d,
-                 dm.n_shared, dm.dtype == PR2_BF16 ? 1 : 0, out, residual};
+                 dm.n_shared, dm.dtype == PR2_BF16 ? 1 : 0, out, residual, status};
   err = launch_combine(ca, num_sms, st);
   mark(events ? events->end : nullptr);
   if (err == cudaSuccess && counts != nullptr)

@@ -531,6 +531,174 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+// ---- combine through shared memory (bf16) ---------------------------------------------------
+// out[t] = round(residual[t] + sum_s g[t,s] Y[inv[t,s]] + sum_j Ys[j,t]), the same arithmetic in
+// the same order as combine_kernel.  Persistent, one CTA per SM, tokens t = blockIdx.x + i *
+// gridDim.x.  Warp 0 is the producer: for each token it copies the token's rows (its k expert
+// rows, its shared-expert rows and the residual row) into one slot of a ring in shared memory
+// with 1-D bulk copies, so that a few hundred KB per SM are in flight; warps 1-8 sum a slot,
+// each thread one 16-byte column chunk per pass, and release it.
+constexpr int kCbConsumers = 8;
+constexpr int kCbThreads = 32 * (kCbConsumers + 1);
+constexpr int kCbMaxSlots = 8;
+constexpr int kCbAhead = 4;  // tokens whose route entries the producer holds in advance
+constexpr int kCbDataBytes = 196 * 1024;  // ring of token slots
+constexpr int kCbSmemBytes = 128 + kCbDataBytes + kCbMaxSlots * (32 * 4 + 8) + 2 * kCbMaxSlots * 8;
+
+struct CombineRing {
+  int slots, rows, row_bytes;
+};
+
+__host__ __device__ inline CombineRing combine_ring(int k, int d, int n_shared, bool residual) {
+  CombineRing r;
+  r.rows = k + n_shared + (residual ? 1 : 0);
+  r.row_bytes = d * 2;
+  const int64_t slot = static_cast<int64_t>(r.rows) * r.row_bytes;
+  const int64_t n = slot > 0 ? kCbDataBytes / slot : 0;
+  r.slots = static_cast<int>(n < kCbMaxSlots ? n : kCbMaxSlots);
+  return r;
+}
+
+constexpr int kCbMaxK = 8;  // the bf16 layer supports k <= 8
+
+__global__ void __launch_bounds__(kCbThreads, 1)
+    combine_bulk_kernel(const __nv_bfloat16* __restrict__ Y, const __nv_bfloat16* __restrict__ Ys,
+                        const int32_t* __restrict__ inv, const float* __restrict__ gates,
+                        int64_t Tn, int k, int d, int n_shared, const __nv_bfloat16* residual,
+                        __nv_bfloat16* out, int32_t* status) {
+  extern __shared__ uint8_t cb_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(cb_raw) + 127) & ~static_cast<uintptr_t>(127));
+  const CombineRing ring = combine_ring(k, d, n_shared, residual != nullptr);
+  const int S = ring.slots;
+  const int slot_bytes = ring.rows * ring.row_bytes;
+  float* meta_gate = reinterpret_cast<float*>(base + kCbDataBytes);             // [S][32]
+  uint32_t* meta_mask = reinterpret_cast<uint32_t*>(meta_gate + kCbMaxSlots * 32);  // [S]
+  uint64_t* full = reinterpret_cast<uint64_t*>(
+      (reinterpret_cast<uintptr_t>(meta_mask + kCbMaxSlots) + 7) & ~static_cast<uintptr_t>(7));
+  uint64_t* empty = full + kCbMaxSlots;
+  __shared__ int abort_flag_s;
+  volatile int* abort_flag = &abort_flag_s;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], kCbConsumers);
+    }
+    abort_flag_s = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  pdl_wait();
+  pdl_trigger();
+  const int nvec = d / 8;
+  if (warp == 0) {
+    // ---------------- producer ----------------
+    uint32_t issued = 0, last_par = 0;
+    int slot = 0;
+    uint32_t phase = 0;
+    // route entries of this CTA's next kCbAhead tokens, loaded ahead so that no token waits
+    // for a global-memory round trip before its copies are issued (lane s: slot s)
+    int q_pos[kCbAhead];
+    float q_g[kCbAhead];
+    auto fetch = [&](int64_t tt, int& p, float& gg) {
+      p = -1;
+      gg = 0.f;
+      if (lane < k && tt < Tn) {
+        p = inv[tt * k + lane];
+        gg = gates[tt * k + lane];
+      }
+    };
+#pragma unroll
+    for (int j = 0; j < kCbAhead; ++j) fetch(blockIdx.x + int64_t{j} * gridDim.x, q_pos[j], q_g[j]);
+    for (int64_t t = blockIdx.x; t < Tn; t += gridDim.x) {
+      const int pos = q_pos[0];
+      const float gt = q_g[0];
+#pragma unroll
+      for (int j = 0; j + 1 < kCbAhead; ++j) {
+        q_pos[j] = q_pos[j + 1];
+        q_g[j] = q_g[j + 1];
+      }
+      fetch(t + int64_t{kCbAhead} * gridDim.x, q_pos[kCbAhead - 1], q_g[kCbAhead - 1]);
+      if (!mbar_wait(&empty[slot], phase ^ 1u, abort_flag, status)) break;
+      const uint32_t vmask = __ballot_sync(0xffffffffu, pos >= 0);
+      if (lane < k) meta_gate[slot * 32 + lane] = gt;
+      if (lane == 0) meta_mask[slot] = vmask;
+      __syncwarp();
+      const uint32_t nrows = __popc(vmask) + n_shared + (residual != nullptr ? 1 : 0);
+      const uint32_t dst = smem_u32(base + slot * slot_bytes);
+      const uint32_t rb = static_cast<uint32_t>(ring.row_bytes);
+      if (lane == 0) mbar_arrive_expect_tx(&full[slot], nrows * rb);  // releases the meta data
+      __syncwarp();
+      if (pos >= 0) bulk_load(dst + lane * rb, Y + static_cast<int64_t>(pos) * d, rb, &full[slot]);
+      if (lane < n_shared)
+        bulk_load(dst + (k + lane) * rb, Ys + (static_cast<int64_t>(lane) * Tn + t) * d, rb,
+                  &full[slot]);
+      if (lane == 0 && residual != nullptr)
+        bulk_load(dst + (k + n_shared) * rb, residual + t * d, rb, &full[slot]);
+      issued |= 1u << slot;
+      last_par = (last_par & ~(1u << slot)) | (phase << slot);
+      if (++slot == S) {
+        slot = 0;
+        phase ^= 1u;
+      }
+    }
+    // no copy may still be landing when the CTA leaves (the consumers may have given up)
+    if (lane == 0)
+      for (int s = 0; s < S; ++s)
+        if ((issued >> s) & 1u)
+          mbar_wait_slow(&full[s], (last_par >> s) & 1u, nullptr, nullptr, kDrainLimitNs);
+  } else {
+    // ---------------- consumers ----------------
+    const int ct = threadIdx.x - 32;
+    int slot = 0;
+    uint32_t phase = 0;
+    for (int64_t t = blockIdx.x; t < Tn; t += gridDim.x) {
+      if (!mbar_wait(&full[slot], phase, abort_flag, status)) break;
+      const uint8_t* sbase = base + slot * slot_bytes;
+      const uint32_t vmask = meta_mask[slot];
+      const float* gs = meta_gate + slot * 32;
+      for (int c = ct; c < nvec; c += 32 * kCbConsumers) {
+        float acc[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[j] = 0.f;
+        if (residual != nullptr) {
+          const uint4 r = reinterpret_cast<const uint4*>(sbase + (k + n_shared) * ring.row_bytes)[c];
+          const __nv_bfloat16* v = reinterpret_cast<const __nv_bfloat16*>(&r);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) acc[j] = __bfloat162float(v[j]);
+        }
+#pragma unroll
+        for (int s = 0; s < kCbMaxK; ++s) {
+          if (s >= k || !((vmask >> s) & 1u)) continue;
+          const uint4 r = reinterpret_cast<const uint4*>(sbase + s * ring.row_bytes)[c];
+          const __nv_bfloat16* v = reinterpret_cast<const __nv_bfloat16*>(&r);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) acc[j] = fmaf(gs[s], __bfloat162float(v[j]), acc[j]);
+        }
+        for (int j2 = 0; j2 < n_shared; ++j2) {
+          const uint4 r = reinterpret_cast<const uint4*>(sbase + (k + j2) * ring.row_bytes)[c];
+          const __nv_bfloat16* v = reinterpret_cast<const __nv_bfloat16*>(&r);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) acc[j] += __bfloat162float(v[j]);
+        }
+        uint4 o;
+        o.x = pack_bf16x2(acc[0], acc[1]);
+        o.y = pack_bf16x2(acc[2], acc[3]);
+        o.z = pack_bf16x2(acc[4], acc[5]);
+        o.w = pack_bf16x2(acc[6], acc[7]);
+        reinterpret_cast<uint4*>(out + t * d)[c] = o;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[slot]);
+      if (++slot == S) {
+        slot = 0;
+        phase ^= 1u;
+      }
+    }
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st) {
@@ -596,6 +764,19 @@ cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st) {
     auto* Ys = static_cast<const __nv_bfloat16*>(a.Ys);
     auto* out = static_cast<__nv_bfloat16*>(a.out);
     auto* res = static_cast<const __nv_bfloat16*>(a.residual);
+    const CombineRing ring = combine_ring(a.k, a.d, a.n_shared, res != nullptr);
+    const bool aligned = ((reinterpret_cast<uintptr_t>(res) | reinterpret_cast<uintptr_t>(Y) |
+                           reinterpret_cast<uintptr_t>(Ys)) & 15u) == 0;
+    if (ring.slots >= 3 && a.k <= kCbMaxK && a.n_shared <= 32 && (a.d * 2) % 16 == 0 &&
+        aligned) {
+      const int ctas = static_cast<int>(a.T < num_sms ? a.T : num_sms);
+      auto* kern = combine_bulk_kernel;
+      const cudaError_t err =
+          cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kCbSmemBytes);
+      if (err != cudaSuccess) return err;
+      return launch_pdl(kern, dim3(ctas), dim3(kCbThreads), kCbSmemBytes, st, 1, Y, Ys, a.inv,
+                        a.gates, a.T, a.k, a.d, a.n_shared, res, out, a.status);
+    }
     return a.k <= 8 ? launch_pdl(combine_kernel<__nv_bfloat16, 8, 8>, grid, block, 0, st, 1, Y,
                                  Ys, a.inv, a.gates, a.T, a.k, a.d, a.n_shared, res, out)
                     : launch_pdl(combine_kernel<__nv_bfloat16, 8, 32>, grid, block, 0, st, 1, Y,

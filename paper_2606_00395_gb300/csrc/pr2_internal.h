@@ -117,6 +117,7 @@ struct CombineArgs {
   int k, d, n_shared, bf16;
   void* out;            // [T, d]
   const void* residual; // [T, d] added to the sum (nullable); may equal `out`
+  int32_t* status;      // PR2_STATUS_TIMEOUT if a bounded wait ran out (nullable)
 };
 cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st);
 
