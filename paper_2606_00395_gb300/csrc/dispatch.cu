@@ -597,8 +597,9 @@ __global__ void __launch_bounds__(kCbThreads, 1)
     uint32_t issued = 0, last_par = 0;
     int slot = 0;
     uint32_t phase = 0;
-    // route entries of this CTA's next kCbAhead tokens, loaded ahead so that no token waits
-    // for a global-memory round trip before its copies are issued (lane s: slot s)
+    // Route entries of this CTA's next kCbAhead tokens, loaded ahead so that no token waits for
+    // a global-memory round trip before its copies are issued (lane s: slot s).  The token loop
+    // is unrolled by kCbAhead, so entry j is read kCbAhead tokens after its load was issued.
     int q_pos[kCbAhead];
     float q_g[kCbAhead];
     auto fetch = [&](int64_t tt, int& p, float& gg) {
@@ -609,38 +610,44 @@ __global__ void __launch_bounds__(kCbThreads, 1)
         gg = gates[tt * k + lane];
       }
     };
+    const int64_t stride = gridDim.x;
 #pragma unroll
-    for (int j = 0; j < kCbAhead; ++j) fetch(blockIdx.x + int64_t{j} * gridDim.x, q_pos[j], q_g[j]);
-    for (int64_t t = blockIdx.x; t < Tn; t += gridDim.x) {
-      const int pos = q_pos[0];
-      const float gt = q_g[0];
+    for (int j = 0; j < kCbAhead; ++j) fetch(blockIdx.x + j * stride, q_pos[j], q_g[j]);
+    bool ok = true;
+    for (int64_t t0 = blockIdx.x; t0 < Tn && ok; t0 += kCbAhead * stride) {
 #pragma unroll
-      for (int j = 0; j + 1 < kCbAhead; ++j) {
-        q_pos[j] = q_pos[j + 1];
-        q_g[j] = q_g[j + 1];
-      }
-      fetch(t + int64_t{kCbAhead} * gridDim.x, q_pos[kCbAhead - 1], q_g[kCbAhead - 1]);
-      if (!mbar_wait(&empty[slot], phase ^ 1u, abort_flag, status)) break;
-      const uint32_t vmask = __ballot_sync(0xffffffffu, pos >= 0);
-      if (lane < k) meta_gate[slot * 32 + lane] = gt;
-      if (lane == 0) meta_mask[slot] = vmask;
-      __syncwarp();
-      const uint32_t nrows = __popc(vmask) + n_shared + (residual != nullptr ? 1 : 0);
-      const uint32_t dst = smem_u32(base + slot * slot_bytes);
-      const uint32_t rb = static_cast<uint32_t>(ring.row_bytes);
-      if (lane == 0) mbar_arrive_expect_tx(&full[slot], nrows * rb);  // releases the meta data
-      __syncwarp();
-      if (pos >= 0) bulk_load(dst + lane * rb, Y + static_cast<int64_t>(pos) * d, rb, &full[slot]);
-      if (lane < n_shared)
-        bulk_load(dst + (k + lane) * rb, Ys + (static_cast<int64_t>(lane) * Tn + t) * d, rb,
-                  &full[slot]);
-      if (lane == 0 && residual != nullptr)
-        bulk_load(dst + (k + n_shared) * rb, residual + t * d, rb, &full[slot]);
-      issued |= 1u << slot;
-      last_par = (last_par & ~(1u << slot)) | (phase << slot);
-      if (++slot == S) {
-        slot = 0;
-        phase ^= 1u;
+      for (int j = 0; j < kCbAhead; ++j) {
+        const int64_t t = t0 + j * stride;
+        if (t >= Tn || !ok) break;
+        const int pos = q_pos[j];
+        const float gt = q_g[j];
+        fetch(t + kCbAhead * stride, q_pos[j], q_g[j]);
+        if (!mbar_wait(&empty[slot], phase ^ 1u, abort_flag, status)) {
+          ok = false;
+          break;
+        }
+        const uint32_t vmask = __ballot_sync(0xffffffffu, pos >= 0);
+        if (lane < k) meta_gate[slot * 32 + lane] = gt;
+        if (lane == 0) meta_mask[slot] = vmask;
+        __syncwarp();
+        const uint32_t nrows = __popc(vmask) + n_shared + (residual != nullptr ? 1 : 0);
+        const uint32_t dst = smem_u32(base + slot * slot_bytes);
+        const uint32_t rb = static_cast<uint32_t>(ring.row_bytes);
+        if (lane == 0) mbar_arrive_expect_tx(&full[slot], nrows * rb);  // releases the meta data
+        __syncwarp();
+        if (pos >= 0)
+          bulk_load(dst + lane * rb, Y + static_cast<int64_t>(pos) * d, rb, &full[slot]);
+        if (lane < n_shared)
+          bulk_load(dst + (k + lane) * rb, Ys + (static_cast<int64_t>(lane) * Tn + t) * d, rb,
+                    &full[slot]);
+        if (lane == 0 && residual != nullptr)
+          bulk_load(dst + (k + n_shared) * rb, residual + t * d, rb, &full[slot]);
+        issued |= 1u << slot;
+        last_par = (last_par & ~(1u << slot)) | (phase << slot);
+        if (++slot == S) {
+          slot = 0;
+          phase ^= 1u;
+        }
       }
     }
     // no copy may still be landing when the CTA leaves (the consumers may have given up)
