@@ -107,7 +107,8 @@ pr2_status pr2_route_replay(const pr2_dims* dims, const void* h, const void* W_r
  * at that point of the launch sequence.  NULL members and a NULL struct pointer are ignored. */
 typedef struct {
     void* start;         /* before dispatch                                              */
-    void* dispatched;    /* after histogram, scan, stable placement and row gather       */
+    void* dispatched;    /* after histogram, scan and stable placement (+ the row gather
+                          * on the fp32 path; the bf16 gate/up GEMM gathers its rows)    */
     void* gate_up_done;  /* after the gate/up + SwiGLU GEMM(s) (routed, then shared)     */
     void* down_done;     /* after the down GEMM(s)                                       */
     void* end;           /* after the gate-weighted combine                              */
