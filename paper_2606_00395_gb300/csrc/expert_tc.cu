@@ -86,21 +86,34 @@ __device__ __forceinline__ void gather_a_producer(const GemmArgs& g, uint8_t* sm
   const __nv_bfloat16* h = static_cast<const __nv_bfloat16*>(g.a_src);
   const int64_t ld = g.K;
   const uint64_t keep = l2_policy_evict_last();  // h: every token row is read k times
-  int stage = 0;
-  ReleaseCursor rel;
-  bool ok = true;
-  for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
-    const TileEntry te = g.tiles[tile / n_tiles_n];
-    const __nv_bfloat16* src[8];
-    uint32_t nbytes[8];
+  // Row pointers of a tile: token perm[a_row0 + row] / k of h; padding rows are zero-filled
+  // (nothing is read).  The next tile's entry and pointers are fetched while the current tile
+  // streams, so no tile starts with two dependent global-memory round trips.
+  const int stride = static_cast<int>(gridDim.x);
+  auto entry = [&](int tile) {
+    return tile < num_tiles ? g.tiles[tile / n_tiles_n] : TileEntry{0, 0, 0, 0};
+  };
+  auto rows_of = [&](const TileEntry& te, const __nv_bfloat16* (&src)[8], uint32_t& live) {
+    live = 0;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const int row = r0 + 16 * i;
-      const bool live = row < te.rows;
-      const int64_t t = live ? g.perm[te.a_row0 + row] / g.k : 0;
-      src[i] = h + t * ld + c * 8;  // padding rows: zero-filled, nothing read
-      nbytes[i] = live ? 16u : 0u;
+      const bool on = row < te.rows;
+      const int64_t t = on ? g.perm[te.a_row0 + row] / g.k : 0;
+      src[i] = h + t * ld + c * 8;
+      live |= (on ? 1u : 0u) << i;
     }
+  };
+  const __nv_bfloat16* src[8];
+  const __nv_bfloat16* src_next[8];
+  uint32_t live = 0, live_next = 0;
+  rows_of(entry(blockIdx.x), src, live);
+  TileEntry te_next = entry(blockIdx.x + stride);
+  const int kb_fetch = KB > 2 ? 2 : KB - 1;  // by then te_next has landed
+  int stage = 0;
+  ReleaseCursor rel;
+  bool ok = true;
+  for (int tile = blockIdx.x; tile < num_tiles && ok; tile += stride) {
     for (int kb = 0; kb < KB; ++kb) {
       if (!rel.wait(empty_b, abort_flag, g.status)) {
         ok = false;
@@ -110,10 +123,15 @@ __device__ __forceinline__ void gather_a_producer(const GemmArgs& g, uint8_t* sm
       const uint32_t dst = smem_u32(smem + stage * kATile) + soff;
 #pragma unroll
       for (int i = 0; i < 8; ++i)
-        cp_async_16_hint(dst + i * 2048, src[i] + kb * kBK, nbytes[i], keep);
+        cp_async_16_hint(dst + i * 2048, src[i] + kb * kBK, ((live >> i) & 1u) * 16u, keep);
       cp_async_arrive_noinc(&full_a[stage]);
       if (++stage == kStagesA) stage = 0;
+      if (kb == kb_fetch) rows_of(te_next, src_next, live_next);
     }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) src[i] = src_next[i];
+    live = live_next;
+    te_next = entry(tile + 2 * stride);
   }
   cp_async_commit();
   cp_async_wait<0>();  // nothing may still be writing shared memory when the CTA leaves
@@ -185,10 +203,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     // same time, so they take the normal L2 policy (an evict_last hint on them pushes out h,
     // H and Y, which later tiles and kernels read again).
     bool ok = true;
+    // the next tile's entry is loaded while this tile streams
+    TileEntry te_next = g.tiles[blockIdx.x / n_tiles_n];
     for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
       const int mt = tile / n_tiles_n;
       const int nt = tile - mt * n_tiles_n;
-      const TileEntry te = g.tiles[mt];
+      const TileEntry te = te_next;
+      const int nxt = tile + static_cast<int>(gridDim.x);
+      if (nxt < num_tiles) te_next = g.tiles[nxt / n_tiles_n];
       const int brow = te.expert * g.b_rows_per_expert + nt * kColsPerTile;
       for (int kb = 0; kb < KB; ++kb) {
         const bool free = is_a ? rel.wait(empty_b, abort_flag, g.status)
