@@ -10,14 +10,16 @@
 // CTAs running at the same time share the weight tiles of the same few experts through L2.
 // The A rows and the expert weight tiles (streamed from DRAM) travel in two separate rings of
 // 128-byte-swizzled K-major tiles (A 4 x 16 KB, B 5 x 32 KB), so the long-latency weight stream
-// runs further ahead of the tensor core.  Warp roles:
-//   warps 0-3  A producers.  Gate/up GEMM of the routed experts: all 128 threads gather the
+// runs further ahead of the tensor core.  Warp roles (warp w runs on SM sub-partition w % 4):
+//   warps 0-2, 4  A producers.  Gate/up GEMM of the routed experts: all 128 threads gather the
 //              tile's rows straight from h with 16-byte cp.async (each thread owns 8 rows and
 //              one 16-byte column chunk, written to its swizzled position), so neither a
 //              permuted copy of h nor a gather launch exists; h (T x d) stays in L2.  Other
-//              GEMMs: one thread issues TMA loads of the A tile.
-//   warp 4     TMEM owner and tcgen05.mma issuer (M=128, N=256, K=16) into one of two
-//              256-column fp32 accumulators.
+//              GEMMs: one thread of warp 0 issues TMA loads of the A tile.
+//   warp 3     TMEM owner and tcgen05.mma issuer (M=128, N=256, K=16) into one of two
+//              256-column fp32 accumulators.  It shares its sub-partition with one epilogue
+//              warp only: next to a gather warp as well it issued late enough to cost the
+//              gate/up GEMM 4 %.
 //   warp 5     TMA producer of the weight ring.
 //   warps 6-9  epilogue: drain the other accumulator (one thread per tile row) while the next
 //              tile is being multiplied.
@@ -32,13 +34,13 @@ namespace pr2 {
 namespace {
 
 constexpr int kThreads = 320;
-constexpr int kWarpMma = 4;
+constexpr int kWarpMma = 3;
 constexpr int kWarpB = 5;
 constexpr int kBK = 64;
 constexpr int kBN = 256;
 constexpr int kStagesA = 4;
 constexpr int kStagesB = 5;
-constexpr int kGatherThreads = 128;         // warps 0-3
+constexpr int kGatherThreads = 128;         // warps 0-2 and 4
 constexpr int kATile = kTileM * kBK * 2;    // 16 KB
 constexpr int kBTile = kBN * kBK * 2;       // 32 KB
 constexpr int kBRing = kStagesA * kATile;   // offset of the B ring
@@ -69,7 +71,7 @@ struct ReleaseCursor {
   }
 };
 
-// A producer of the gathered gate/up GEMM: thread `tid` of warps 0-3 copies, for every K block,
+// A producer of the gathered gate/up GEMM: thread `tid` of warps 0-2, 4 copies, for every K block,
 // the 16-byte chunk `c = tid % 8` of tile rows r = tid / 8 + 16 i (i = 0..7).  In the 128-byte
 // swizzled K-major tile, chunk c of row r sits at r * 128 + ((c ^ (r % 8)) * 16), and r % 8 is
 // the same for all eight rows of a thread.  After its eight copies of a stage the thread
@@ -79,7 +81,7 @@ __device__ __forceinline__ void gather_a_producer(const GemmArgs& g, uint8_t* sm
                                                   uint64_t* full_a, uint64_t* empty_b,
                                                   volatile int* abort_flag, int n_tiles_n,
                                                   int num_tiles, int KB) {
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x < 96 ? threadIdx.x : threadIdx.x - 32;  // warps 0-2, 4
   const int c = tid & 7;
   const int r0 = tid >> 3;
   const uint32_t soff = static_cast<uint32_t>(r0 * 128 + ((c ^ (r0 & 7)) << 4));
@@ -188,7 +190,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_trigger();
   const int num_tiles = (*g.num_tiles) * n_tiles_n;
 
-  if (kGatherA && warp < 4) {
+  if (kGatherA && (warp < 3 || warp == 4)) {
     gather_a_producer(g, smem, full_a, empty_b, abort_flag, n_tiles_n, num_tiles, KB);
   } else if ((warp == 0 || warp == kWarpB) && lane == 0) {
     // ---------------- TMA producers: warp 0 the A ring, warp 5 the B ring ----------------
