@@ -9,8 +9,8 @@
 // Persistent kernel: one CTA per SM walks the (M-tile, N-tile) list in M-major order, so the
 // CTAs running at the same time share the weight tiles of the same few experts through L2.
 // The A rows and the expert weight tiles (streamed from DRAM) travel in two separate rings of
-// 128-byte-swizzled K-major tiles (A 4 x 16 KB, B 5 x 32 KB), so the long-latency weight stream
-// runs further ahead of the tensor core.  Warp roles (warp w runs on SM sub-partition w % 4):
+// 128-byte-swizzled K-major tiles (A 4 x 16 KB, B 5 x 32 KB), each filled by its own producers,
+// so the long-latency weight stream runs further ahead of the tensor core.  Warp roles (warp w runs on SM sub-partition w % 4):
 //   warps 0-2, 4  A producers.  Gate/up GEMM of the routed experts: all 128 threads gather the
 //              tile's rows straight from h with 16-byte cp.async (each thread owns 8 rows and
 //              one 16-byte column chunk, written to its swizzled position), so neither a
@@ -24,9 +24,7 @@
 //   warps 6-9  epilogue: drain the other accumulator (one thread per tile row) while the next
 //              tile is being multiplied.
 // Each tcgen05.commit costs the tensor pipe about 25 ns (a third of one MMA), so the MMA thread
-// commits once per K block, to the weight ring's empty barrier.  That completion also frees the
-// A stage the K block used: the A producers wait on the weight ring's barrier of the K block
-// kStagesA earlier instead of on a barrier of their own.
+// commits once per K block, to one release barrier shared by both rings (ReleaseCursor).
 #include "pr2_device.cuh"
 #include "pr2_internal.h"
 
@@ -38,47 +36,49 @@ constexpr int kWarpMma = 3;
 constexpr int kWarpB = 5;
 constexpr int kBK = 64;
 constexpr int kBN = 256;
-constexpr int kStagesA = 4;
-constexpr int kStagesB = 5;
 constexpr int kGatherThreads = 128;         // warps 0-2 and 4
 constexpr int kATile = kTileM * kBK * 2;    // 16 KB
 constexpr int kBTile = kBN * kBK * 2;       // 32 KB
-constexpr int kBRing = kStagesA * kATile;   // offset of the B ring
 constexpr int kAccCols = kBN;               // one accumulator
 constexpr uint32_t kTmemCols = 2 * kAccCols;
+constexpr int kRel = 8;                     // release barriers, one per K block mod 8
+
+constexpr int kStagesA = 4;                 // 4 x 16 KB A ring + 5 x 32 KB weight ring = 224 KB
+constexpr int kStagesB = 5;
+constexpr int kBRing = kStagesA * kATile;   // offset of the weight ring
 constexpr int kBarOffset = kBRing + kStagesB * kBTile;
 constexpr int kSmemBytes = 1024 + kBarOffset + 256;
-// The A producer's wait on empty_b relies on that barrier never being two phases ahead of it.
-static_assert(kStagesA <= kStagesB, "the A ring may not be deeper than the weight ring");
+static_assert(kStagesA < kRel && kStagesB < kRel, "a ring of kRel stages could see a release twice");
+static_assert((kStagesA + kStagesB + kRel + 5) * 8 + 8 <= 256, "barrier area");
 
-// Where the A producer learns that an A stage is free: K block n reuses the A stage of K block
-// j = n - kStagesA, whose MMAs completed phase j / kStagesB of empty_b[j % kStagesB].
+// Stage release.  The MMA thread commits once per K block (each tcgen05.commit costs the tensor
+// pipe ~25 ns, a third of an MMA), to rel[n % kRel] for the n-th K block.  A producer whose ring
+// has S stages may refill the stage of K block n once K block n - S has completed, i.e. phase
+// (n - S) / kRel of rel[(n - S) % kRel].  That barrier cannot be a phase further on: its next
+// completion is K block n - S + kRel, whose data this producer has not issued yet (S < kRel).
+template <int S>
 struct ReleaseCursor {
-  int n = 0;          // K blocks issued so far
-  int slot = 0;       // empty_b slot of K block n - kStagesA
-  uint32_t par = 0;   // its phase parity
-  __device__ __forceinline__ bool wait(uint64_t* empty_b, volatile int* abort_flag,
-                                       int32_t* status) {
-    if (n < kStagesA) return true;
-    return mbar_wait(&empty_b[slot], par, abort_flag, status);
+  int n = 0;  // K blocks issued so far
+  __device__ __forceinline__ bool wait(uint64_t* rel, volatile int* abort_flag, int32_t* status) {
+    if (n < S) return true;
+    const int j = n - S;
+    return mbar_wait(&rel[j % kRel], static_cast<uint32_t>(j / kRel) & 1u, abort_flag, status);
   }
-  __device__ __forceinline__ void advance() {
-    if (n++ < kStagesA) return;
-    if (++slot == kStagesB) {
-      slot = 0;
-      par ^= 1u;
-    }
-  }
+  __device__ __forceinline__ void advance() { ++n; }
 };
 
-// A producer of the gathered gate/up GEMM: thread `tid` of warps 0-2, 4 copies, for every K block,
-// the 16-byte chunk `c = tid % 8` of tile rows r = tid / 8 + 16 i (i = 0..7).  In the 128-byte
-// swizzled K-major tile, chunk c of row r sits at r * 128 + ((c ^ (r % 8)) * 16), and r % 8 is
-// the same for all eight rows of a thread.  After its eight copies of a stage the thread
+// A producer of the gathered gate/up GEMM: thread `tid` of warps 0-2, 4 copies, for every K
+// block, the 16-byte chunk `c = tid % 8` of tile rows r = tid / 8 + 16 i (i = 0..7).  In the
+// 128-byte swizzled K-major tile, chunk c of row r sits at r * 128 + ((c ^ (r % 8)) * 16), and
+// r % 8 is the same for all eight rows of a thread.  After its eight copies of a stage the thread
 // registers an arrival on that stage's full barrier (count 128) that fires when they have
 // landed; the MMA thread, after acquiring the barrier, fences the stage into the async proxy.
+// A tile's rows are tokens perm[a_row0 + r] / k of h.  The next tile's table entry is loaded
+// when a tile starts and its perm entries halfway through the tile, as raw values that are
+// only turned into pointers when the next tile starts: no load result is waited for while the
+// ring needs refilling.
 __device__ __forceinline__ void gather_a_producer(const GemmArgs& g, uint8_t* smem,
-                                                  uint64_t* full_a, uint64_t* empty_b,
+                                                  uint64_t* full_a, uint64_t* rel_bar,
                                                   volatile int* abort_flag, int n_tiles_n,
                                                   int num_tiles, int KB) {
   const int tid = threadIdx.x < 96 ? threadIdx.x : threadIdx.x - 32;  // warps 0-2, 4
@@ -88,52 +88,52 @@ __device__ __forceinline__ void gather_a_producer(const GemmArgs& g, uint8_t* sm
   const __nv_bfloat16* h = static_cast<const __nv_bfloat16*>(g.a_src);
   const int64_t ld = g.K;
   const uint64_t keep = l2_policy_evict_last();  // h: every token row is read k times
-  // Row pointers of a tile: token perm[a_row0 + row] / k of h; padding rows are zero-filled
-  // (nothing is read).  The next tile's entry and pointers are fetched while the current tile
-  // streams, so no tile starts with two dependent global-memory round trips.
   const int stride = static_cast<int>(gridDim.x);
   auto entry = [&](int tile) {
     return tile < num_tiles ? g.tiles[tile / n_tiles_n] : TileEntry{0, 0, 0, 0};
   };
-  auto rows_of = [&](const TileEntry& te, const __nv_bfloat16* (&src)[8], uint32_t& live) {
+  // perm entries of a tile's rows (padding rows: none, they are zero-filled)
+  auto fetch = [&](const TileEntry& te, int32_t (&slot)[8], uint32_t& live) {
     live = 0;
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const int row = r0 + 16 * i;
       const bool on = row < te.rows;
-      const int64_t t = on ? g.perm[te.a_row0 + row] / g.k : 0;
-      src[i] = h + t * ld + c * 8;
+      slot[i] = on ? g.perm[te.a_row0 + row] : 0;
       live |= (on ? 1u : 0u) << i;
     }
   };
-  const __nv_bfloat16* src[8];
-  const __nv_bfloat16* src_next[8];
+  int32_t slot[8], slot_next[8];
   uint32_t live = 0, live_next = 0;
-  rows_of(entry(blockIdx.x), src, live);
+  fetch(entry(blockIdx.x), slot, live);
   TileEntry te_next = entry(blockIdx.x + stride);
-  const int kb_fetch = KB > 2 ? 2 : KB - 1;  // by then te_next has landed
+  const int kb_fetch = KB / 2;
   int stage = 0;
-  ReleaseCursor rel;
+  ReleaseCursor<kStagesA> rc;
   bool ok = true;
   for (int tile = blockIdx.x; tile < num_tiles && ok; tile += stride) {
+    const __nv_bfloat16* src[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) src[i] = h + static_cast<int64_t>(slot[i] / g.k) * ld + c * 8;
+    const TileEntry te_after = entry(tile + 2 * stride);  // used by the next tile's fetch
     for (int kb = 0; kb < KB; ++kb) {
-      if (!rel.wait(empty_b, abort_flag, g.status)) {
+      if (!rc.wait(rel_bar, abort_flag, g.status)) {
         ok = false;
         break;
       }
-      rel.advance();
+      rc.advance();
       const uint32_t dst = smem_u32(smem + stage * kATile) + soff;
 #pragma unroll
       for (int i = 0; i < 8; ++i)
         cp_async_16_hint(dst + i * 2048, src[i] + kb * kBK, ((live >> i) & 1u) * 16u, keep);
       cp_async_arrive_noinc(&full_a[stage]);
       if (++stage == kStagesA) stage = 0;
-      if (kb == kb_fetch) rows_of(te_next, src_next, live_next);
+      if (kb == kb_fetch) fetch(te_next, slot_next, live_next);
     }
 #pragma unroll
-    for (int i = 0; i < 8; ++i) src[i] = src_next[i];
+    for (int i = 0; i < 8; ++i) slot[i] = slot_next[i];
     live = live_next;
-    te_next = entry(tile + 2 * stride);
+    te_next = te_after;
   }
   cp_async_commit();
   cp_async_wait<0>();  // nothing may still be writing shared memory when the CTA leaves
@@ -149,8 +149,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* full_a = reinterpret_cast<uint64_t*>(smem + kBarOffset);
   uint64_t* full_b = full_a + kStagesA;
-  uint64_t* empty_b = full_b + kStagesB;
-  uint64_t* acc_full = empty_b + kStagesB;  // [2]
+  uint64_t* rel = full_b + kStagesB;         // [kRel]
+  uint64_t* acc_full = rel + kRel;           // [2]
   uint64_t* acc_empty = acc_full + 2;    // [2]
   uint64_t* drain = acc_empty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
@@ -164,10 +164,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStagesA; ++s) mbar_init(&full_a[s], kGatherA ? kGatherThreads : 1);
-    for (int s = 0; s < kStagesB; ++s) {
-      mbar_init(&full_b[s], 1);
-      mbar_init(&empty_b[s], 1);
-    }
+    for (int s = 0; s < kStagesB; ++s) mbar_init(&full_b[s], 1);
+    for (int s = 0; s < kRel; ++s) mbar_init(&rel[s], 1);
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
       mbar_init(&acc_empty[b], 4);  // one arrival per epilogue warp
@@ -191,7 +189,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int num_tiles = (*g.num_tiles) * n_tiles_n;
 
   if (kGatherA && (warp < 3 || warp == 4)) {
-    gather_a_producer(g, smem, full_a, empty_b, abort_flag, n_tiles_n, num_tiles, KB);
+    gather_a_producer(g, smem, full_a, rel, abort_flag, n_tiles_n, num_tiles, KB);
   } else if ((warp == 0 || warp == kWarpB) && lane == 0) {
     // ---------------- TMA producers: warp 0 the A ring, warp 5 the B ring ----------------
     const bool is_a = warp == 0;
@@ -200,7 +198,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t issued = 0, last_par = 0;
     int stage = 0;
     uint32_t phase = 0;
-    ReleaseCursor rel;  // A ring: stage release through the weight ring's barriers
+    ReleaseCursor<kStagesA> rca;
+    ReleaseCursor<kStagesB> rcb;
     // Expert weights are reused only by the M-tiles of their expert, which run at about the
     // same time, so they take the normal L2 policy (an evict_last hint on them pushes out h,
     // H and Y, which later tiles and kernels read again).
@@ -215,14 +214,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (nxt < num_tiles) te_next = g.tiles[nxt / n_tiles_n];
       const int brow = te.expert * g.b_rows_per_expert + nt * kColsPerTile;
       for (int kb = 0; kb < KB; ++kb) {
-        const bool free = is_a ? rel.wait(empty_b, abort_flag, g.status)
-                               : mbar_wait(&empty_b[stage], phase ^ 1u, abort_flag, g.status);
+        const bool free = is_a ? rca.wait(rel, abort_flag, g.status)
+                               : rcb.wait(rel, abort_flag, g.status);
         if (!free) {
           ok = false;
           break;
         }
+        rca.advance();
+        rcb.advance();
         if (is_a) {
-          rel.advance();
           uint8_t* sa = smem + stage * kATile;
           mbar_arrive_expect_tx(&fullr[stage], kATile);
           tma_load_2d(sa, &tm_a, &fullr[stage], kb * kBK, te.a_row0);
@@ -250,6 +250,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t pha = 0, phb = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
+    int kn = 0;  // K blocks issued: K block kn releases through rel[kn % kRel]
     bool ok = true;
     for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
       if (!mbar_wait(&acc_empty[acc], acc_phase ^ 1u, abort_flag, g.status)) break;
@@ -269,7 +270,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kk = 0; kk < kBK / 16; ++kk)
           umma_bf16(d_tmem, umma_desc_sw128(sa + kk * 32), umma_desc_sw128(sb + kk * 32), idesc,
                     (kb > 0 || kk > 0) ? 1u : 0u);
-        umma_commit(&empty_b[sb_i]);  // frees this K block's weight stage and A stage
+        umma_commit(&rel[kn % kRel]);  // frees this K block's A and weight stages
+        ++kn;
         if (++sa_i == kStagesA) {
           sa_i = 0;
           pha ^= 1u;
