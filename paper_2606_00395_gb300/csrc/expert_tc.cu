@@ -325,9 +325,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const float h1 = __fdividef(g1, 1.0f + __expf(-g1)) * u1;
               pk[j] = pack_bf16x2(h0, h1);
             }
-            uint4* dst = reinterpret_cast<uint4*>(orow + col);
-            dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+            st_global_v8(orow + col, pk);  // 16 columns = one 32-byte sector
           }
         }
       } else {
@@ -342,9 +340,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int j = 0; j < 8; ++j)
               pk[j] = pack_bf16x2(__uint_as_float(rv[2 * j]), __uint_as_float(rv[2 * j + 1]));
-            uint4* dst = reinterpret_cast<uint4*>(orow + col);
-            dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+            st_global_v8(orow + col, pk);  // 16 columns = one 32-byte sector
           }
         }
       }
