@@ -406,7 +406,7 @@ def run_pr2(args, rank, world, local_rank):
     bsets = [make_evs(True) for _ in range(n_break)]
     run(n_break, bsets)
     torch.cuda.synchronize()
-    per = dict(step=[], route_predict=[], route_replay=[], dispatch=[], gate_up=[], down=[],
+    per = dict(step=[], route_predict=[], route_replay=[], dispatch=[], expert_gemm=[],
                combine=[], layer_rollout=[], layer_replay=[])
     for e in bsets:
         per["step"].append(el(e[0], e[6]))
@@ -416,8 +416,8 @@ def run_pr2(args, rank, world, local_rank):
         per["layer_replay"].append(el(e[3], e[6]))
         for _, st in (e[2], e[5]):
             per["dispatch"].append(el(st[0], st[1]))
-            per["gate_up"].append(el(st[1], st[2]))
-            per["down"].append(el(st[2], st[3]))
+            # routed gate/up and down run as one launch (plus the shared experts' GEMMs)
+            per["expert_gemm"].append(el(st[1], st[3]))
             per["combine"].append(el(st[3], st[4]))
     value = replicas.job_throughput(cfg.T * args.steps, world, total_ms)
     mean = {k: statistics.mean(v) for k, v in per.items()}
@@ -434,17 +434,14 @@ def run_pr2(args, rank, world, local_rank):
         "route_predict": cost.route_predict_work(cfg.T, cfg.d, cfg.N, cfg.k, cfg.dtype, True),
         "route_replay": cost.route_replay_work(cfg.T, cfg.d, cfg.N, cfg.k, cfg.dtype, False),
         "dispatch": cost.dispatch_work(cfg.T, cfg.d, cfg.k, cfg.dtype, gather=cfg.dtype == "fp32"),
-        "gate_up": cost.expert_gate_up_work(F, cfg.d, cfg.m, hit, cfg.dtype,
+        "expert_gemm": cost.expert_mlp_work(F, cfg.d, cfg.m, hit, cfg.dtype,
                                             a_rows=cfg.T if cfg.dtype == "bf16" else None),
-        "down": cost.expert_down_work(F, cfg.d, cfg.m, hit, cfg.dtype),
         "combine": cost.combine_work(cfg.T, cfg.d, cfg.k, cfg.n_shared, cfg.dtype),
     }
     if cfg.n_shared:
-        sg = cost.expert_gate_up_work(cfg.T * cfg.n_shared, cfg.d, cfg.m, cfg.n_shared, cfg.dtype)
-        sd = cost.expert_down_work(cfg.T * cfg.n_shared, cfg.d, cfg.m, cfg.n_shared, cfg.dtype)
-        work["gate_up"] = cost.KernelWork(work["gate_up"].bytes + sg.bytes,
-                                          work["gate_up"].flops + sg.flops)
-        work["down"] = cost.KernelWork(work["down"].bytes + sd.bytes, work["down"].flops + sd.flops)
+        sw = cost.expert_mlp_work(cfg.T * cfg.n_shared, cfg.d, cfg.m, cfg.n_shared, cfg.dtype)
+        work["expert_gemm"] = cost.KernelWork(work["expert_gemm"].bytes + sw.bytes,
+                                              work["expert_gemm"].flops + sw.flops)
     kernels = {}
     for name, w in work.items():
         ms = mean[name]
@@ -458,14 +455,22 @@ def run_pr2(args, rank, world, local_rank):
             kernels[name] = dict(ms=ms, bound="hbm", achieved=w.bytes / (ms * 1e-3) / 1e9,
                                  peak=pk["hbm"], unit="GB/s", frac=t_hbm / ms,
                                  algorithmic_flops=w.flops, algorithmic_bytes=w.bytes)
-    dom = max(("gate_up", "down"), key=lambda n: kernels[n]["ms"])
+    dom = "expert_gemm"
     dk = kernels[dom]
-    roofline = dict(kernel=f"expert_tc_kernel ({dom})", bound=dk["bound"], achieved=dk["achieved"],
+    # The tensor-core fraction of the grouped GEMM, beside its binding (HBM) bound: against the
+    # burst bf16 peak (a GEMM timed alone) and the sustained one (a GEMM inside a long run of
+    # steps under the power cap, as here).
+    dk["tensor_frac"] = work[dom].flops / (pk["bf16"] * 1e12) * 1e3 / dk["ms"]
+    dk["tensor_frac_sustained"] = work[dom].flops / (pk["bf16_sustained"] * 1e12) * 1e3 / dk["ms"]
+    roofline = dict(kernel="expert_tc_kernel (routed gate/up + down, one launch)",
+                    bound=dk["bound"], achieved=dk["achieved"],
                     peak=dk["peak"], unit=dk["unit"], frac=dk["frac"],
                     traffic=measured_traffic(f"{cfg.name}/{dom}"),
                     peak_source=f"{pk['source']} (MEASURED_PEAKS.json burst)"
                     if pk["source"] == "measured" else "fallback",
                     algorithmic=("flops" if dk["bound"] == "tensor" else "bytes"),
+                    tensor_frac=dk["tensor_frac"],
+                    tensor_frac_sustained=dk["tensor_frac_sustained"],
                     per_launch_units=f"{F} token-expert rows x (d={cfg.d}, m={cfg.m})")
 
     extras = measure_extras(cfg, L, W2, dm, flush, pk, iters=args.extras_iters)
@@ -545,10 +550,12 @@ def run_pr2(args, rank, world, local_rank):
 
     # per layer forward: dispatch (one fused cooperative kernel when N % 4 == 0 and the grid is
     # resident, as at every bench shape; else hist + scan + place; + a row gather on the fp32
-    # path only, the bf16 gate/up GEMM gathers its A rows itself), the two grouped GEMMs (+ two
-    # for shared experts) and the combine; plus one routing kernel per mode
+    # path only, the bf16 gate/up GEMM gathers its A rows itself), the routed grouped GEMMs (one
+    # launch for gate/up and down in bf16, two in fp32; + two for shared experts) and the
+    # combine; plus one routing kernel per mode
     n_dispatch = (1 if cfg.N % 4 == 0 and cfg.N <= 256 else 3) + (cfg.dtype == "fp32")
-    launches_per_step = 2 + 2 * (n_dispatch + 3 + (2 if cfg.n_shared else 0))
+    n_gemm = 1 if cfg.dtype == "bf16" else 2
+    launches_per_step = 2 + 2 * (n_dispatch + n_gemm + 1 + (2 if cfg.n_shared else 0))
     line = dict(metric=METRIC, value=value, unit="tokens/s", n_gpus=world, steps=args.steps,
                 warmup=args.warmup, ms_per_step=total_ms / args.steps, higher_is_better=True,
                 scaling="weak", vs_baseline=None, dtype=cfg.dtype, data="synthetic",

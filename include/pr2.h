@@ -109,8 +109,10 @@ typedef struct {
     void* start;         /* before dispatch                                              */
     void* dispatched;    /* after histogram, scan and stable placement (+ the row gather
                           * on the fp32 path; the bf16 gate/up GEMM gathers its rows)    */
-    void* gate_up_done;  /* after the gate/up + SwiGLU GEMM(s) (routed, then shared)     */
-    void* down_done;     /* after the down GEMM(s)                                       */
+    void* gate_up_done;  /* after the routed experts' GEMMs (bf16: gate/up and down run as
+                          * one launch) and the shared experts' gate/up GEMM              */
+    void* down_done;     /* after the shared experts' down GEMM (the routed down GEMM on
+                          * the fp32 path)                                               */
     void* end;           /* after the gate-weighted combine                              */
 } pr2_stage_events;
 

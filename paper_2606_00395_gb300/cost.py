@@ -89,6 +89,14 @@ def expert_down_work(rows: int, d: int, m: int, experts_hit: int,
     return KernelWork(rows * m * e + experts_hit * d * m * e + rows * d * e, 2 * rows * m * d)
 
 
+def expert_mlp_work(rows: int, d: int, m: int, experts_hit: int, dtype: str = "bf16",
+                    a_rows: int | None = None) -> KernelWork:
+    """Both grouped GEMMs of the gated MLP (gate/up + SwiGLU, then down), run as one launch."""
+    g = expert_gate_up_work(rows, d, m, experts_hit, dtype, a_rows)
+    dn = expert_down_work(rows, d, m, experts_hit, dtype)
+    return KernelWork(g.bytes + dn.bytes, g.flops + dn.flops)
+
+
 def combine_work(T: int, d: int, k: int, n_shared: int = 0, dtype: str = "bf16") -> KernelWork:
     """out[t] = sum_s g[t,s] Y[inv[t,s]] (+ shared rows): read Y, gates, inv; write out."""
     e = _esz(dtype)

@@ -78,6 +78,7 @@ struct Workspace {
   int32_t* inv;
   int32_t* num_tiles;
   unsigned int* sync_ctr;
+  int32_t* ready;
   TileEntry* tiles;
   TileEntry* stiles1;
   TileEntry* stiles2;
@@ -112,6 +113,7 @@ Workspace carve(const pr2_dims& dm, uint8_t* base) {
   w.inv = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * F));
   w.num_tiles = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * 2));
   w.sync_ctr = reinterpret_cast<unsigned int*>(take(sizeof(unsigned int)));
+  w.ready = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * w.max_tiles));
   w.tiles = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * w.max_tiles));
   w.stiles1 = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * (w.shared_tiles + 1)));
   w.stiles2 = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * (w.shared_tiles + 1)));
@@ -419,7 +421,8 @@ pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* 
   const int es = static_cast<int>(esize(dm));
   DispatchArgs da{idx,       dm.T,       dm.k,      dm.N,    dm.d,   es,     dm.n_shared,
                   w.blk_hist, w.counts,  w.offsets, w.perm,  w.inv,  w.tiles, w.num_tiles,
-                  w.stiles1, w.stiles2,  h,         w.xperm, status, w.sync_ctr};
+                  w.stiles1, w.stiles2,  h,         w.xperm, status, w.sync_ctr,
+                  dm.dtype == PR2_BF16 ? w.ready : nullptr};
   // (w.xperm is nullptr on the bf16 path: dispatch then launches no gather)
   if (err == cudaSuccess) err = launch_dispatch(da, num_sms, st);
   mark(events ? events->dispatched : nullptr);
@@ -435,9 +438,8 @@ pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* 
   GemmArgs s2{w.stiles2, w.num_tiles + 1, w.shared_tiles, dm.m, dm.d, dm.d, w.ys, status,
               nullptr, nullptr, 0};
   if (dm.dtype == PR2_BF16) {
-    CUtensorMap a1, b1g, b1u, a2, b2, sa1, sb1g, sb1u, sa2, sb2;
-    bool ok = make_tmap_bf16(&a1, h, dm.d, dm.T, 64, kTileM) &&  // unused: A is gathered
-              make_tmap_bf16(&b1g, W_gate, dm.d, (uint64_t)dm.N * dm.m, 64, 128) &&
+    CUtensorMap b1g, b1u, a2, b2, sa1, sb1g, sb1u, sa2, sb2;
+    bool ok = make_tmap_bf16(&b1g, W_gate, dm.d, (uint64_t)dm.N * dm.m, 64, 128) &&
               make_tmap_bf16(&b1u, W_up, dm.d, (uint64_t)dm.N * dm.m, 64, 128) &&
               make_tmap_bf16(&a2, w.hbuf, dm.m, F, 64, kTileM) &&
               make_tmap_bf16(&b2, W_down, dm.m, (uint64_t)dm.N * dm.d, 64, 256);
@@ -449,13 +451,18 @@ pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* 
            make_tmap_bf16(&sb2, Ws_down, dm.m, (uint64_t)dm.n_shared * dm.d, 64, 256);
     }
     if (!ok) return PR2_ERR_CUDA;
-    err = launch_expert_tc(true, true, a1, b1g, b1u, g1, num_sms, st);
-    if (err == cudaSuccess && dm.n_shared > 0)
-      err = launch_expert_tc(true, false, sa1, sb1g, sb1u, s1, num_sms, st);
+    // routed experts: gate/up then down in one cooperative launch
+    MlpArgs routed{{g1, g2}, w.ready};
+    err = launch_expert_tc(kExpertFused, a2, b1g, b1u, b2, routed, num_sms, st);
+    if (err == cudaSuccess && dm.n_shared > 0) {
+      MlpArgs sh1{{s1, s1}, nullptr};
+      err = launch_expert_tc(kExpertGateUpTma, sa1, sb1g, sb1u, sb1g, sh1, num_sms, st);
+    }
     mark(events ? events->gate_up_done : nullptr);
-    if (err == cudaSuccess) err = launch_expert_tc(false, false, a2, b2, b2, g2, num_sms, st);
-    if (err == cudaSuccess && dm.n_shared > 0)
-      err = launch_expert_tc(false, false, sa2, sb2, sb2, s2, num_sms, st);
+    if (err == cudaSuccess && dm.n_shared > 0) {
+      MlpArgs sh2{{s2, s2}, nullptr};
+      err = launch_expert_tc(kExpertDown, sa2, sb2, sb2, sb2, sh2, num_sms, st);
+    }
     mark(events ? events->down_done : nullptr);
   } else {
     err = launch_expert_simt(true, static_cast<const float*>(w.xperm),

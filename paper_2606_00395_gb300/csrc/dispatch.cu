@@ -95,7 +95,8 @@ __global__ void __launch_bounds__(1024)
     scan_kernel(int32_t* __restrict__ blk_hist, int nblk, int N, int64_t T, int n_shared,
                 int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
                 TileEntry* __restrict__ tiles, int32_t* __restrict__ num_tiles,
-                TileEntry* __restrict__ stiles1, TileEntry* __restrict__ stiles2) {
+                TileEntry* __restrict__ stiles1, TileEntry* __restrict__ stiles2,
+                int32_t* __restrict__ ready) {
   __shared__ int sh[32];
   __shared__ int part[1024];  // [G][N_pad] partial sums, then their exclusive scan over g
   __shared__ int ex_off[kMaxExpertsDispatch + 1];
@@ -176,6 +177,7 @@ __global__ void __launch_bounds__(1024)
     const int r0 = ex_off[lo] + j * kTileM;
     const int left = ex_off[lo + 1] - r0;
     tiles[i] = TileEntry{lo, r0, left < kTileM ? left : kTileM, r0};
+    if (ready != nullptr) ready[i] = 0;  // per M-tile counter of the fused expert GEMM
   }
   // Shared experts: every token, fixed tiles.  Gate/up reads h rows, down reads Hs rows.
   const int mt_T = static_cast<int>((T + kTileM - 1) / kTileM);
@@ -262,7 +264,7 @@ __global__ void __launch_bounds__(kDispatchChunk)
                           int32_t* __restrict__ inv, TileEntry* __restrict__ tiles,
                           int32_t* __restrict__ num_tiles, TileEntry* __restrict__ stiles1,
                           TileEntry* __restrict__ stiles2, unsigned int* sync_ctr,
-                          int32_t* status) {
+                          int32_t* status, int32_t* __restrict__ ready) {
   extern __shared__ int dsm[];
   int* wcnt = dsm;                   // [kWarps][N] per-warp counts, then per-warp bases
   int* tot = wcnt + kWarps * N;      // [N] slots of each expert over all blocks
@@ -385,6 +387,7 @@ __global__ void __launch_bounds__(kDispatchChunk)
       const int r0 = ex_off[lo] + j * kTileM;
       const int left = ex_off[lo + 1] - r0;
       tiles[i] = TileEntry{lo, r0, left < kTileM ? left : kTileM, r0};
+      if (ready != nullptr) ready[i] = 0;  // per M-tile counter of the fused expert GEMM
     }
     const int mt_T = static_cast<int>((T + kTileM - 1) / kTileM);
     for (int i = tid; i < n_shared * mt_T; i += blockDim.x) {
@@ -727,7 +730,7 @@ cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st)
     cfg.numAttrs = 1;
     err = cudaLaunchKernelEx(&cfg, dispatch_fused_kernel, a.idx, F, a.k, a.N, a.T, a.n_shared,
                              a.blk_hist, a.counts, a.offsets, a.perm, a.inv, a.tiles,
-                             a.num_tiles, a.stiles1, a.stiles2, a.sync_ctr, a.status);
+                             a.num_tiles, a.stiles1, a.stiles2, a.sync_ctr, a.status, a.ready);
     if (err != cudaSuccess) return err;
   } else {
     if (nblk > 0) {
@@ -737,7 +740,7 @@ cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st)
     }
     err = launch_pdl(scan_kernel, dim3(1), dim3(1024), 0, st, 1, a.blk_hist, nblk, a.N, a.T,
                      a.n_shared, a.counts, a.offsets, a.tiles, a.num_tiles, a.stiles1,
-                     a.stiles2);
+                     a.stiles2, a.ready);
     if (err != cudaSuccess) return err;
     if (nblk > 0) {
       err = launch_pdl(place_kernel, dim3(nblk), dim3(kDispatchChunk), 0, st, 1, a.idx, F, a.k,

@@ -105,6 +105,8 @@ struct DispatchArgs {
   void* xperm;           // [T*k, d] permuted copy of h (fp32 path); nullptr: no gather launch
   int32_t* status;
   unsigned int* sync_ctr;  // grid-barrier counter of the fused dispatch (zeroed per call)
+  int32_t* ready;          // [max_mtiles] per M-tile counters of the fused GEMM, cleared here
+                           // (nullable)
 };
 cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st);
 
@@ -138,11 +140,23 @@ struct GemmArgs {
   const int32_t* perm;
   int k;
 };
-// swiglu: out = silu(A Wg^T) * (A Wu^T) (tm_b0 = gate, tm_b1 = up); else out = A Wb^T.
-// gather_a: A rows are read from g.a_src through g.perm (tm_a unused); else from tm_a.
-cudaError_t launch_expert_tc(bool swiglu, bool gather_a, const CUtensorMap& tm_a,
-                             const CUtensorMap& tm_b0, const CUtensorMap& tm_b1,
-                             const GemmArgs& g, int num_sms, cudaStream_t st);
+// Launch kinds of the tcgen05 grouped GEMM (expert_tc.cu).  Phase 0 is a gate/up GEMM with the
+// SwiGLU epilogue (weights tm_b0 = gate, tm_b1 = up), phase 1 a down GEMM (weights tm_b2).
+enum ExpertKind : int {
+  kExpertGateUpGather = 0,  // phase 0, A rows gathered from p[0].a_src through p[0].perm
+  kExpertGateUpTma = 1,     // phase 0, A rows from tm_a (shared experts: rows of h)
+  kExpertDown = 2,          // phase 1, A rows from tm_a
+  kExpertFused = 3,         // phase 0 (gathered) then phase 1 (A = p[0].out through tm_a) in
+                            // one cooperative launch
+};
+struct MlpArgs {
+  GemmArgs p[2];     // arguments of phase 0 and phase 1 (only the launched phases are read)
+  int32_t* ready;    // kExpertFused: per M-tile count of finished gate/up epilogue warps,
+                     // zero on entry (dispatch clears it)
+};
+cudaError_t launch_expert_tc(ExpertKind kind, const CUtensorMap& tm_a, const CUtensorMap& tm_b0,
+                             const CUtensorMap& tm_b1, const CUtensorMap& tm_b2,
+                             const MlpArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_expert_simt(bool swiglu, const float* A, const float* Wb0, const float* Wb1,
                                const GemmArgs& g, cudaStream_t st);
 

@@ -35,6 +35,8 @@ def test_kernel_work_counts_each_tensor_once():
     # gathering A from h: each of the 4096 tokens crosses HBM once instead of k = 8 times
     gg = cost.expert_gate_up_work(32768, 2048, 768, 128, a_rows=4096)
     assert g.bytes - gg.bytes == (32768 - 4096) * 2048 * 2 and gg.flops == g.flops
+    mlp = cost.expert_mlp_work(32768, 2048, 768, 128, a_rows=4096)
+    assert mlp.bytes == gg.bytes + dn.bytes and mlp.flops == g.flops + dn.flops
     assert cost.dispatch_work(4096, 2048, 8).bytes == 3 * 4096 * 8 * 4
     assert (cost.dispatch_work(4096, 2048, 8, "fp32", gather=True).bytes
             == 3 * 4096 * 8 * 4 + 4096 * 2048 * 4 + 32768 * 2048 * 4)
