@@ -55,6 +55,7 @@ typedef enum { PR2_FP32 = 0, PR2_BF16 = 1 } pr2_dtype;
 /* dims->flags bits */
 #define PR2_F_SYNC_STATUS 0x1u /* synchronise `stream` and turn the status word into a code */
 #define PR2_F_DELTA_LOSS 0x2u  /* pr2_predictor_loss: the delta-matching variant              */
+#define PR2_F_NORMALIZE_TOPK 0x4u /* routing: gates renormalised over the selected experts    */
 
 /* device status word bits (OR-ed in by the kernels; the caller zeroes the word) */
 #define PR2_STATUS_BAD_INDEX 0x1
@@ -81,7 +82,9 @@ typedef struct {
  *  W_router   [N, d]  dtype     old-snapshot router (transposed W_old)
  *  W_pred     [N, d]  dtype     evolution predictor (transposed W_p)
  *  idx        [T, k]  int32     out: I_hat, slots by descending rho_hat, ties to the lower index
- *  gates      [T, k]  fp32      out: rho_hat at idx (full-softmax probability, not renormalised)
+ *  gates      [T, k]  fp32      out: rho_hat at idx (full-softmax probability; divided by its
+ *                               sum over the k slots only with PR2_F_NORMALIZE_TOPK in dims->flags,
+ *                               the Qwen3 reading: the paper weights with rho_hat itself)
  *  logits_old [T, N]  fp32      out, nullable: p_old, the feature-cache logits of Algorithm 2
  *  near_tie   [1]     int64     in/out, nullable: += #tokens whose rho_hat_(k) - rho_hat_(k+1)
  *                               < PR2_NEAR_TIE_GAP (k < N)
@@ -95,7 +98,8 @@ pr2_status pr2_route_predict(const pr2_dims* dims, const void* h, const void* W_
  * Training-time replay gates, Sec. 4.1 "Replay During Training" (Algorithm 3, first step):
  *     rho = Softmax(h W),  gates[t,s] = rho[t, idx[t,s]];  no fresh top-k, no predictor.
  *  h [T,d], W_router [N,d] (current router, dtype); idx [T,k] int32 the cached route;
- *  gates [T,k] fp32 out (0 for an invalid slot); probs [T,N] fp32 out, nullable: the full rho;
+ *  gates [T,k] fp32 out (0 for an invalid slot; with PR2_F_NORMALIZE_TOPK divided by the sum
+ *  over the token's valid slots); probs [T,N] fp32 out, nullable: the full rho (never divided);
  *  status_dev nullable (PR2_STATUS_BAD_INDEX for an index outside [0,N) or repeated in a token).
  */
 pr2_status pr2_route_replay(const pr2_dims* dims, const void* h, const void* W_router,

@@ -17,6 +17,9 @@ Functions (each cites the passage it follows in the C source):
 * ``feature_cache``  - the fixed-length feature cache of Algorithm 2 (evenly spaced positions)
 * ``rollout_layers`` - Algorithm 2 over L stacked layers with the residual stream (composition
   of ``route_predict`` and ``moe_forward``)
+* ``normalize_topk`` - the optional renormalisation of the selected gates (g / sum g, as in
+  Qwen3's router).  The paper weights with the probabilities themselves (Eqs. pr2_old_output /
+  pr2_output); this is the reading behind PR2_F_NORMALIZE_TOPK, not part of the method.
 
 Parity status: every function is pinned by the CPU tests in ``tests/test_oracle_pins.py``.
 """
@@ -120,10 +123,19 @@ def _same_dtype(*codes):
     return codes[0]
 
 
-def route_predict(h, W_router, W_pred, k: int, lib=None):
+def normalize_topk(gates):
+    """Selected gates divided by their sum per token (fp64); a row whose gates are all zero (every
+    slot invalid) stays zero."""
+    g = np.asarray(gates, dtype=np.float64)
+    s = g.sum(axis=1, keepdims=True)
+    return np.divide(g, s, out=np.zeros_like(g), where=s > 0)
+
+
+def route_predict(h, W_router, W_pred, k: int, lib=None, normalize: bool = False):
     """Rollout routing of Sec. 4.1 in fp64.  Returns a dict of numpy arrays:
     idx [T,k] int32, gates [T,k], logits [T,N] (= p_old), probs [T,N] (= rho-hat),
-    margin [T] (= rho-hat_(k) - rho-hat_(k+1)), top_vals [T,k+1]."""
+    margin [T] (= rho-hat_(k) - rho-hat_(k+1)), top_vals [T,k+1].  ``normalize``: gates
+    renormalised over the route (``normalize_topk``); probs, margin and top_vals are not."""
     hs, c0 = _stored(h)
     ws, c1 = _stored(W_router)
     ps, c2 = _stored(W_pred)
@@ -138,11 +150,14 @@ def route_predict(h, W_router, W_pred, k: int, lib=None):
     _load(lib).oracle_route_predict(T, d, N, k, dt, _ptr(hs), _ptr(ws), _ptr(ps), _ptr(out["idx"]),
                                  _ptr(out["gates"]), _ptr(out["logits"]), _ptr(out["probs"]),
                                  _ptr(out["margin"]), _ptr(out["top_vals"]))
+    if normalize:
+        out["gates"] = normalize_topk(out["gates"])
     return out
 
 
-def route_replay(h, W_router, idx, lib=None):
-    """Replay gates of Sec. 4.1 in fp64: dict(gates [T,k], probs [T,N], bad = #invalid slots)."""
+def route_replay(h, W_router, idx, lib=None, normalize: bool = False):
+    """Replay gates of Sec. 4.1 in fp64: dict(gates [T,k], probs [T,N], bad = #invalid slots).
+    ``normalize``: gates renormalised over the valid slots (``normalize_topk``)."""
     hs, c0 = _stored(h)
     ws, c1 = _stored(W_router)
     dt = _same_dtype(c0, c1)
@@ -154,6 +169,8 @@ def route_replay(h, W_router, idx, lib=None):
     probs = np.zeros((T, N))
     bad = _load(lib).oracle_route_replay(T, d, N, k, dt, _ptr(hs), _ptr(ws), _ptr(ix), _ptr(gates),
                                       _ptr(probs))
+    if normalize:
+        gates = normalize_topk(gates)
     return dict(gates=gates, probs=probs, bad=int(bad))
 
 

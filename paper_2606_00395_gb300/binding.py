@@ -24,6 +24,7 @@ PR2_OK = 0
 PR2_FP32, PR2_BF16 = 0, 1
 PR2_F_SYNC_STATUS = 0x1
 PR2_F_DELTA_LOSS = 0x2
+PR2_F_NORMALIZE_TOPK = 0x4
 PR2_STATUS_BAD_INDEX = 0x1
 PR2_STATUS_TIMEOUT = 0x2
 PR2_NEAR_TIE_GAP = 1e-4

@@ -186,6 +186,7 @@ pr2_status route_common(const pr2_dims* dims, bool predict, const void* h, const
     a.logits_or_probs = aux;
     a.near_tie = near_tie;
     a.status = status_dev;
+    a.norm = (dm.flags & PR2_F_NORMALIZE_TOPK) ? 1 : 0;
     err = launch_route_tc(mode, tm_h, tm_w, tm_wp, a, split, st);
   }
   return finish(err, dm.flags, status_dev, st);

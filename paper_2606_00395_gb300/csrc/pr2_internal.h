@@ -71,6 +71,7 @@ struct RouteTcArgs {
   float* logits_or_probs;  // predict: p_old [T,N]; replay: rho [T,N]; nullable
   int64_t* near_tie;
   int32_t* status;
+  int norm;                // PR2_F_NORMALIZE_TOPK: gates divided by their sum over the route
   // kModeLoss only (h = h_old, W = W_p)
   const float* p_old;      // [T, N] cached router logits
   const float* rho;        // [T_rho, N] teacher probabilities

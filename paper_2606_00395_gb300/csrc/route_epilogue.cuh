@@ -49,8 +49,10 @@ __device__ __forceinline__ bool route_warp_finish(bool predict, int64_t t, int N
                                                   const int32_t* __restrict__ idx_in,
                                                   int32_t* __restrict__ idx_out,
                                                   float* __restrict__ gates,
-                                                  float* __restrict__ aux, int32_t* status) {
+                                                  float* __restrict__ aux, int32_t* status,
+                                                  bool norm) {
   const int lane = threadIdx.x & 31;
+  float gsum = 0.f;  // sum of the written gates (lane 0), for PR2_F_NORMALIZE_TOPK
   float mx = -FLT_MAX;
 #pragma unroll
   for (int j = 0; j < kRoutePerLane; ++j) mx = fmaxf(mx, zr[j]);
@@ -94,6 +96,7 @@ __device__ __forceinline__ bool route_warp_finish(bool predict, int64_t t, int N
         if (lane == 0) {
           idx_out[t * k + r] = bi;
           gates[t * k + r] = prob;
+          gsum += prob;
         }
         prev = prob;
       } else {
@@ -113,10 +116,16 @@ __device__ __forceinline__ bool route_warp_finish(bool predict, int64_t t, int N
         if (j == ej) v = zr[j];
       v = __shfl_sync(0xffffffffu, v, ok ? (e & 31) : 0);
       if (lane == 0) {
-        gates[t * k + sl] = ok ? expf(v - mx) * inv_s : 0.f;
+        const float g = ok ? expf(v - mx) * inv_s : 0.f;
+        gates[t * k + sl] = g;
+        gsum += g;
         if (!ok && status != nullptr) atomicOr(status, PR2_STATUS_BAD_INDEX);
       }
     }
+  }
+  if (norm && lane == 0 && gsum > 0.f) {  // renormalise the row just written (this thread's stores)
+    const float sc = 1.0f / gsum;
+    for (int r = 0; r < k; ++r) gates[t * k + r] *= sc;
   }
   return tie;
 }

@@ -3,6 +3,7 @@
 //   predict (Eqs. pr2_predict, pr2_route): z = h W^T + h W_p^T, rho_hat = Softmax(z),
 //            idx = TopK(rho_hat, k) (ties to the lower expert), gates = rho_hat[idx].
 //   replay  (Sec. 4.1 "Replay During Training"): rho = Softmax(h W^T), gates = rho[idx_in].
+// PR2_F_NORMALIZE_TOPK divides a token's gates by their sum (over its valid slots).
 #include <float.h>
 
 #include "route_epilogue.cuh"
@@ -17,7 +18,7 @@ __global__ void __launch_bounds__(kWarps * 32)
                       const float* __restrict__ W, const float* __restrict__ Wp,
                       const int32_t* __restrict__ idx_in, int32_t* __restrict__ idx_out,
                       float* __restrict__ gates, float* __restrict__ aux,
-                      unsigned long long* near_tie, int32_t* status) {
+                      unsigned long long* near_tie, int32_t* status, int norm) {
   pdl_wait();
   pdl_trigger();
   const int lane = threadIdx.x & 31;
@@ -55,7 +56,7 @@ __global__ void __launch_bounds__(kWarps * 32)
     }
   }
   const bool tie = route_warp_finish(predict != 0, t, N, k, zr, pr, idx_in, idx_out, gates, aux,
-                                     status);
+                                     status, norm != 0);
   if (tie && lane == 0 && near_tie != nullptr) atomicAdd(near_tie, 1ull);
 }
 
@@ -70,7 +71,8 @@ cudaError_t launch_route_simt(const pr2_dims& dm, bool predict, const float* h, 
   dim3 grid((T + kWarps - 1) / kWarps);
   return launch_pdl(route_simt_kernel, grid, dim3(kWarps * 32), 0, st, 1, T, dm.d, dm.N, dm.k,
                     predict ? 1 : 0, h, W, Wp, idx_in, idx_out, gates, aux,
-                    reinterpret_cast<unsigned long long*>(near_tie), status);
+                    reinterpret_cast<unsigned long long*>(near_tie), status,
+                    (dm.flags & PR2_F_NORMALIZE_TOPK) ? 1 : 0);
 }
 
 }  // namespace pr2

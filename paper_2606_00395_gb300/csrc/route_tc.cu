@@ -128,22 +128,30 @@ __device__ __forceinline__ int key_e(uint64_t key) {
   return static_cast<int>(~static_cast<uint32_t>(key));
 }
 
-// Write a finished predict row: idx and gates of the k best keys; returns the near-tie flag
-// rho_hat_(k) - rho_hat_(k+1) < PR2_NEAR_TIE_GAP.
+// Write a finished predict row: idx and gates of the k best keys (divided by their sum under
+// PR2_F_NORMALIZE_TOPK); returns the near-tie flag rho_hat_(k) - rho_hat_(k+1) <
+// PR2_NEAR_TIE_GAP, always on the unnormalised probabilities.
 __device__ __forceinline__ bool predict_write(const uint64_t (&key)[16], float mx, float inv_s,
                                               int64_t t, const RouteTcArgs& a) {
   int32_t* irow = a.idx_out + t * a.k;
   float* grow = a.gates + t * a.k;
+  float pr[kKeep];
+  float sk = 0.f;
+#pragma unroll
+  for (int j = 0; j < kKeep; ++j) {
+    pr[j] = expf(key_z(key[j]) - mx) * inv_s;
+    if (j < a.k) sk += pr[j];
+  }
+  const float sc = a.norm ? 1.0f / sk : 1.0f;
   float pk = 0.f, pk1 = 0.f;
 #pragma unroll
   for (int j = 0; j < kKeep; ++j) {
-    const float pr = expf(key_z(key[j]) - mx) * inv_s;
     if (j < a.k) {
       irow[j] = key_e(key[j]);
-      grow[j] = pr;
+      grow[j] = pr[j] * sc;
     }
-    if (j == a.k - 1) pk = pr;
-    if (j == a.k) pk1 = pr;
+    if (j == a.k - 1) pk = pr[j];
+    if (j == a.k) pk1 = pr[j];
   }
   return (a.k < a.N) && (pk - pk1 < (float)PR2_NEAR_TIE_GAP);
 }
@@ -450,9 +458,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int o = 1; o < split; o <<= 1) z_s[s] += __shfl_xor_sync(0xffffffffu, z_s[s], o);
       if (have && live && part == 0) {
         float* grow = a.gates + t * k;
+        float gv[kMaxTopK];
+        float sk = 0.f;
+#pragma unroll
+        for (int s = 0; s < kMaxTopK; ++s) {
+          gv[s] = (s < k && e_s[s] >= 0) ? expf(z_s[s] - mx) * inv_s : 0.f;
+          sk += gv[s];
+        }
+        const float sc = (a.norm && sk > 0.f) ? 1.0f / sk : 1.0f;  // over the valid slots
 #pragma unroll
         for (int s = 0; s < kMaxTopK; ++s)
-          if (s < k) grow[s] = (e_s[s] >= 0) ? expf(z_s[s] - mx) * inv_s : 0.f;
+          if (s < k) grow[s] = gv[s] * sc;
         if (bad && a.status != nullptr) atomicOr(a.status, PR2_STATUS_BAD_INDEX);
       }
       if (have && a.logits_or_probs != nullptr) {

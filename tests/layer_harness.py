@@ -31,8 +31,8 @@ def to_dev(L, dev="cuda"):
     return {k: (v.to(dev) if v is not None else None) for k, v in L.items()}
 
 
-def gpu_predict(cfg, Ld, logits=True, stream=None):
-    dm = dims_of(cfg)
+def gpu_predict(cfg, Ld, logits=True, stream=None, flags=0):
+    dm = dims_of(cfg, flags)
     idx, gates, aux = B.alloc_route(dm, logits=logits)
     near = torch.zeros(1, dtype=torch.int64, device="cuda")
     status = torch.zeros(1, dtype=torch.int32, device="cuda")
@@ -41,8 +41,8 @@ def gpu_predict(cfg, Ld, logits=True, stream=None):
     return dict(idx=idx, gates=gates, logits=aux, near_tie=near, status=status)
 
 
-def gpu_replay(cfg, Ld, W, idx, probs=True, stream=None):
-    dm = dims_of(cfg)
+def gpu_replay(cfg, Ld, W, idx, probs=True, stream=None, flags=0):
+    dm = dims_of(cfg, flags)
     gates = torch.empty(cfg.T, cfg.k, dtype=torch.float32, device="cuda")
     pr = torch.empty(cfg.T, cfg.N, dtype=torch.float32, device="cuda") if probs else None
     status = torch.zeros(1, dtype=torch.int32, device="cuda")

@@ -160,3 +160,29 @@ def test_bounded_wait_reports_timeout_instead_of_hanging():
     assert B.pr2_selftest_wait_timeout(status, 20_000_000) == 0
     torch.cuda.synchronize()
     assert int(status.item()) == B.PR2_STATUS_TIMEOUT
+
+
+@pytest.mark.parametrize("name", ["tiny_fp32", "bf16_multitile", "bf16_shared_n256"])
+def test_normalized_gates_match_the_oracle(name):
+    """PR2_F_NORMALIZE_TOPK: the same routes, gates divided by their sum over the route (replay:
+    over the valid slots), in both modes; logits and probabilities are not renormalised."""
+    cfg = SMALL[name]
+    L = synth.make_layer(cfg, seed=3)
+    Ld = H.to_dev(L)
+    flag = B.PR2_F_NORMALIZE_TOPK
+    g = H.gpu_predict(cfg, Ld, flags=flag)
+    orc = oracle.route_predict(L["x"], L["W_router"], L["W_pred"], cfg.k, normalize=True)
+    H.check_routes(orc, H.cpu(g["idx"]).numpy())
+    gidx = H.cpu(g["idx"]).numpy()
+    keep = orc["margin"] >= H.TIE_GAP
+    gg = H.cpu(g["gates"]).numpy()
+    H.rowwise_close(gg[keep], orc["gates"][keep])
+    assert np.max(np.abs(gg.sum(1) - 1.0)) < 1e-5
+    H.rowwise_close(H.cpu(g["logits"]).numpy(), orc["logits"])
+    idx = orc["idx"].copy()
+    idx[0, 0] = cfg.N  # an invalid slot: excluded from the sum
+    r = H.gpu_replay(cfg, Ld, Ld["W_router"], torch.from_numpy(idx).cuda(), flags=flag)
+    orep = oracle.route_replay(L["x"], L["W_router"], idx, normalize=True)
+    H.rowwise_close(H.cpu(r["gates"]).numpy(), orep["gates"])
+    H.rowwise_close(H.cpu(r["probs"]).numpy(), orep["probs"])
+    assert int(r["status"].item()) & B.PR2_STATUS_BAD_INDEX

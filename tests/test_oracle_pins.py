@@ -124,6 +124,32 @@ def test_replay_gates_gather_current_router_probabilities():
     assert np.array_equal(rep["gates"], np.take_along_axis(rep["probs"], idx, 1))
 
 
+def test_normalized_gates_sum_to_one_and_reduce_in_special_cases():
+    """The optional renormalisation (PR2_F_NORMALIZE_TOPK): each row of selected gates sums to
+    1; k = 1 gives exactly 1; k = N leaves the gates (rho-hat sums to 1 over all experts); a
+    uniform router gives 1/k; invalid replay slots stay 0 and the valid ones sum to 1."""
+    T, d, N, k = 24, 16, 9, 3
+    h, W, Wp = _rand((T, d), 70), _rand((N, d), 71, 0.4), _rand((N, d), 72, 0.4)
+    r = oracle.route_predict(h, W, Wp, k, normalize=True)
+    plain = oracle.route_predict(h, W, Wp, k)
+    assert np.array_equal(r["idx"], plain["idx"]) and np.array_equal(r["probs"], plain["probs"])
+    assert np.max(np.abs(r["gates"].sum(1) - 1.0)) < 1e-14
+    assert np.all(r["gates"] > plain["gates"])  # k < N: the sum of the selected is below 1
+    one = oracle.route_predict(h, W, Wp, 1, normalize=True)
+    assert np.all(one["gates"] == 1.0)
+    full = oracle.route_predict(h, W, Wp, N, normalize=True)
+    assert np.max(np.abs(full["gates"] - np.take_along_axis(full["probs"], full["idx"], 1))) < 1e-14
+    uni = oracle.route_predict(h, torch.zeros(N, d), torch.zeros(N, d), k, normalize=True)
+    assert np.max(np.abs(uni["gates"] - 1.0 / k)) < 1e-15
+    idx = plain["idx"].copy()
+    idx[0, 1] = N            # invalid
+    idx[1, :] = -1           # every slot invalid
+    rep = oracle.route_replay(h, W, idx, normalize=True)
+    assert rep["gates"][0, 1] == 0.0 and abs(rep["gates"][0].sum() - 1.0) < 1e-14
+    assert np.all(rep["gates"][1] == 0.0)
+    assert np.max(np.abs(rep["gates"][2:].sum(1) - 1.0)) < 1e-14
+
+
 def test_replay_flags_invalid_and_duplicate_indices():
     T, d, N = 4, 8, 6
     h, W = _rand((T, d), 62), _rand((N, d), 63)
