@@ -178,8 +178,9 @@ def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
     call, L2 flushed before every call, median of ``iters``) against its own roofline:
     the fixed-length feature-cache writer (Algorithm 2) for T_c = min(2048, T) rows (Table 4's
     Qwen3 cache length), the predictive loss with its W_p gradient over that cache (Eq.
-    pr2_loss, Algorithm 3) and the route-tracking diagnostics of the rollout route against the
-    drifted current router (Sec. 5)."""
+    pr2_loss, Algorithm 3), the route-tracking diagnostics of the rollout route against the
+    drifted current router (Sec. 5), the multi-layer decode loop, the latency of one decode
+    batch (routing alone, and the whole layer) and the Pr^3 step."""
     dev = "cuda"
     Tc = min(2048, cfg.T)
     idx, gates, logits = B.alloc_route(dm, logits=True)
@@ -287,6 +288,29 @@ def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
     report("decode_loop_graph", graph_ms, work, layers=Ld, T=Td, eager_ms=eager_ms,
            tokens_per_s=Td / (graph_ms * 1e-3))
     del Ws, graph
+
+    # The rollout decode batch on its own (T = 256 tokens, one per sequence; rollout mode):
+    # latency of the routing call and of the whole layer (routing + forward), each timed alone
+    # from a flushed L2.
+    xd = L["x"][:Td].contiguous()
+    di, dgt, dlg = B.alloc_route(ddm, logits=True)
+    do = torch.empty(Td, cfg.d, dtype=cfg.torch_dtype, device=dev)
+
+    def route_d():
+        B.check(B.pr2_route_predict(ddm, xd, L["W_router"], L["W_pred"], di, dgt, dlg),
+                "pr2_route_predict")
+
+    def layer_d():
+        route_d()
+        B.check(B.pr2_moe_forward(ddm, xd, di, dgt, L["W_gate"], L["W_up"], L["W_down"],
+                                  L["Ws_gate"], L["Ws_up"], L["Ws_down"], do, workspace=dws,
+                                  status=status), "pr2_moe_forward")
+    ms = timed(route_d)
+    report("decode_route_predict", ms, per_layer[0], T=Td, latency_us=ms * 1e3)
+    ms = timed(layer_d)
+    report("decode_layer", ms, cost.KernelWork(sum(w.bytes for w in per_layer),
+                                              sum(w.flops for w in per_layer)),
+           T=Td, latency_us=ms * 1e3, tokens_per_s=Td / (ms * 1e-3))
 
     # Pr^3 step (App. "Predictive Rollout Routing Replay"): rollout with the predicted route,
     # the log-prob pass replaying it with the snapshot router, the gradient pass replaying it

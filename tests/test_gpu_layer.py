@@ -186,3 +186,26 @@ def test_normalized_gates_match_the_oracle(name):
     H.rowwise_close(H.cpu(r["gates"]).numpy(), orep["gates"])
     H.rowwise_close(H.cpu(r["probs"]).numpy(), orep["probs"])
     assert int(r["status"].item()) & B.PR2_STATUS_BAD_INDEX
+
+
+@pytest.mark.parametrize("n_shared", [0, 1])
+def test_all_invalid_route_gives_the_shared_experts_alone(n_shared):
+    """Every cached index invalid: no routed rows (the grouped GEMM launch has no jobs, every
+    combine slot carries no rows), the status flags it, counts are zero and the output is the
+    shared experts' alone (zero without shared experts)."""
+    cfg = synth.LayerConfig("none", T=150, d=256, N=32, k=4, m=128, n_shared=n_shared)
+    L = synth.make_layer(cfg, seed=9)
+    Ld = H.to_dev(L)
+    idx = np.full((cfg.T, cfg.k), -1, np.int32)
+    idx[:, 1] = cfg.N + 3
+    gates = torch.zeros(cfg.T, cfg.k, dtype=torch.float32, device="cuda")
+    f = H.gpu_forward(cfg, Ld, torch.from_numpy(idx).cuda(), gates)
+    assert f["code"] == 0 and int(f["status"].item()) & B.PR2_STATUS_BAD_INDEX
+    assert int(H.cpu(f["counts"]).sum().item()) == 0
+    want = oracle.moe_forward(L["x"], idx, np.zeros((cfg.T, cfg.k)), L["W_gate"], L["W_up"],
+                              L["W_down"], L["Ws_gate"], L["Ws_up"], L["Ws_down"])
+    got = H.cpu(f["out"]).float().numpy()
+    if n_shared == 0:
+        assert np.all(got == 0.0)
+    else:
+        H.normwise_close(got, want, H.OUT_TOL["bf16"])
