@@ -157,7 +157,7 @@ pr2_status pr2_moe_forward(const pr2_dims* dims, const void* h, const int32_t* i
  * nothing.
  *  - Layers whose pr2_moe_workspace_bytes(dims) exceeds pr2_static_scratch_bytes() are
  *    rejected with PR2_ERR_WORKSPACE before anything is launched (e.g. the Qwen3-shaped layer
- *    up to ~400 tokens fits; a 4096-token batch does not).
+ *    up to 743 tokens fits; a 4096-token batch does not).
  *  - The first call on a device looks up the array's device address (cudaGetSymbolAddress,
  *    with that device current); make that first call before any stream capture.
  *  - All calls on a device share the one array: calls whose kernels overlap on the GPU (other
