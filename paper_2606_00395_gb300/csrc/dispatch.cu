@@ -10,15 +10,19 @@
 //   3. place  - one block per 256 slots again: per-warp counts via __match_any_sync, a scan
 //               over the 8 warps, then rank = popc(lanes below with the same expert):
 //               perm[offsets[e] + r] = f, inv[f] = its position (-1 for an invalid slot).
-//   4. gather - X[p, :] = h[perm[p] / k, :], 16-byte vectors, one warp per row.
+//   4. gather - X[p, :] = h[perm[p] / k, :], 16-byte vectors, one warp per row; fp32 path only
+//               (the bf16 gate/up GEMM reads its rows from h through perm itself).
 // Steps 1-3 normally run as one cooperative launch (dispatch_fused_kernel): every block counts
 // its slots, one bounded grid barrier, then each block derives the expert totals, its own
 // per-expert bases and the expert offsets from the whole block histogram (identical in every
-// block), block 0 writes counts, offsets and the tile tables, and every block places its
-// slots.  Shapes whose grid cannot be resident at once use the three kernels above.
+// block), block 0 writes counts, offsets and the tile tables (and clears the grouped GEMM's
+// per-M-tile readiness counters), and every block places its slots.  Shapes whose grid cannot
+// be resident at once use the three kernels above.
 // Combine (the sums of Eqs. pr2_old_output / pr2_output):
 //   out[t, :] = sum_s gates[t,s] * Y[inv[t*k+s], :] + sum_j Ys[j, t, :], fp32 accumulation,
 //   plus, when given, a residual row r[t, :] (the multi-layer loop's h_l; may alias out).
+//   bf16: combine_bulk_kernel (rows streamed into shared memory with bulk copies); fp32 and
+//   layers whose rows do not fit its ring: combine_kernel (rows through registers).
 #include <mutex>
 
 #include "pr2_device.cuh"
@@ -787,10 +791,9 @@ cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st) {
       return launch_pdl(kern, dim3(ctas), dim3(kCbThreads), kCbSmemBytes, st, 1, Y, Ys, a.inv,
                         a.gates, a.T, a.k, a.d, a.n_shared, res, out, a.status);
     }
-    return a.k <= 8 ? launch_pdl(combine_kernel<__nv_bfloat16, 8, 8>, grid, block, 0, st, 1, Y,
-                                 Ys, a.inv, a.gates, a.T, a.k, a.d, a.n_shared, res, out)
-                    : launch_pdl(combine_kernel<__nv_bfloat16, 8, 32>, grid, block, 0, st, 1, Y,
-                                 Ys, a.inv, a.gates, a.T, a.k, a.d, a.n_shared, res, out);
+    // (bf16 layers have k <= 8, checked at the ABI)
+    return launch_pdl(combine_kernel<__nv_bfloat16, 8, 8>, grid, block, 0, st, 1, Y, Ys, a.inv,
+                      a.gates, a.T, a.k, a.d, a.n_shared, res, out);
   }
   auto* Y = static_cast<const float*>(a.Y);
   auto* Ys = static_cast<const float*>(a.Ys);
