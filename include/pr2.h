@@ -71,7 +71,7 @@ typedef struct {
     int64_t T;
     int32_t d, N, k, m, n_shared;
     int32_t dtype;   /* pr2_dtype */
-    uint32_t flags;  /* PR2_F_* */
+    uint32_t flags;  /* PR2_F_* (any other bit: PR2_ERR_INVALID_ARG) */
 } pr2_dims;
 
 /*

@@ -55,6 +55,8 @@ pr2_status check_dims(const pr2_dims* dm) {
       dm->n_shared < 0)
     return PR2_ERR_INVALID_ARG;
   if (dm->dtype != PR2_FP32 && dm->dtype != PR2_BF16) return PR2_ERR_INVALID_ARG;
+  if (dm->flags & ~(PR2_F_SYNC_STATUS | PR2_F_DELTA_LOSS | PR2_F_NORMALIZE_TOPK))
+    return PR2_ERR_INVALID_ARG;  // an unknown flag is a caller error, not a no-op
   if (dm->T * static_cast<int64_t>(dm->k) > (int64_t{1} << 30)) return PR2_ERR_UNSUPPORTED;
   if (dm->N > kMaxExperts) return PR2_ERR_UNSUPPORTED;
   if (dm->dtype == PR2_FP32) {

@@ -191,3 +191,14 @@ def test_rollout_layers_rejects_bad_arguments(lib):
     sync = list(base)
     sync[0] = ctypes.byref(dms)
     assert lib.pr2_rollout_layers(*sync, fake, ctypes.c_size_t(ws), None, None) == 1
+
+
+def test_unknown_flags_are_rejected(lib):
+    ok = B.dims(64, 2048, 128, 8, 768, flags=B.PR2_F_NORMALIZE_TOPK | B.PR2_F_SYNC_STATUS)
+    assert B.pr2_moe_workspace_bytes(ok) > 0
+    bad = B.dims(64, 2048, 128, 8, 768, flags=0x100)
+    assert B.pr2_moe_workspace_bytes(bad) == 0
+    fake = ctypes.c_void_p(256)
+    code = lib.pr2_route_predict(ctypes.byref(bad), fake, fake, fake, fake, fake, None, None, None,
+                                 None)
+    assert code == 1  # PR2_ERR_INVALID_ARG, before any launch
