@@ -27,6 +27,14 @@ SMALL = {
     # bf16 with a shared expert, N = 256 routed experts (two 256-column MMAs in routing)
     "bf16_shared_n256": synth.LayerConfig("bf16_shared_n256", T=200, d=128, N=256, k=8, m=128,
                                           n_shared=1),
+    # degenerate shapes: one expert (top-1 of 1: the dense SwiGLU MLP, gate 1), top-k over all
+    # experts (no (k+1)-th probability, so no near ties), top-1, and a single token (one row
+    # in every tile of both GEMMs, one combine block)
+    "fp32_one_expert": synth.LayerConfig("fp32_one_expert", T=77, d=64, N=1, k=1, m=96,
+                                         dtype="fp32"),
+    "fp32_k_eq_n": synth.LayerConfig("fp32_k_eq_n", T=100, d=64, N=8, k=8, m=64, dtype="fp32"),
+    "bf16_top1": synth.LayerConfig("bf16_top1", T=257, d=128, N=16, k=1, m=64),
+    "bf16_one_token": synth.LayerConfig("bf16_one_token", T=1, d=256, N=32, k=8, m=128),
 }
 
 
@@ -82,6 +90,54 @@ def _full_layer_check(cfg, seed=0):
 def test_small_layer_matches_oracle_everywhere(name):
     exempt, err = _full_layer_check(SMALL[name])
     print(f"{name}: near-tie tokens {exempt}, output error {err:.2e}")
+
+
+@pytest.mark.parametrize("dtype,N,k", [("bf16", 64, 8), ("bf16", 256, 8), ("fp32", 6, 3),
+                                       ("fp32", 8, 8)])
+def test_all_zero_router_routes_to_the_lowest_experts(dtype, N, k):
+    """W = W_p = 0: every logit is 0 and rho_hat is uniform, so all N probabilities tie exactly.
+    The route is experts 0..k-1 in slot order (ties go to the lower expert), every gate is 1/N,
+    every token is a near tie unless k = N, replay of the route gives the same gates, and the
+    layer output is the uniform 1/N mix of the first k experts."""
+    cfg = synth.LayerConfig("zero", T=300, d=128, N=N, k=k, m=128, dtype=dtype)
+    L = synth.make_layer(cfg, seed=4)
+    L["W_router"] = torch.zeros_like(L["W_router"])
+    L["W_pred"] = torch.zeros_like(L["W_pred"])
+    Ld = H.to_dev(L)
+    g = H.gpu_predict(cfg, Ld)
+    idx = H.cpu(g["idx"]).numpy()
+    assert np.array_equal(idx, np.tile(np.arange(k, dtype=np.int32), (cfg.T, 1)))
+    gates = H.cpu(g["gates"]).numpy().astype(np.float64)
+    assert np.max(np.abs(gates * N - 1.0)) <= 1e-6
+    assert np.all(H.cpu(g["logits"]).numpy() == 0.0)
+    assert int(g["near_tie"].item()) == (cfg.T if k < N else 0)
+    orc = oracle.route_predict(L["x"], L["W_router"], L["W_pred"], k)
+    assert np.array_equal(orc["idx"], idx)
+    r = H.gpu_replay(cfg, Ld, Ld["W_router"], g["idx"])
+    assert torch.max(torch.abs(H.cpu(r["gates"]) - H.cpu(g["gates"]))).item() <= 1e-7
+    f = H.gpu_forward(cfg, Ld, g["idx"], g["gates"])
+    assert f["code"] == 0 and int(f["status"].item()) == 0
+    want = oracle.moe_forward(L["x"], orc["idx"], orc["gates"], L["W_gate"], L["W_up"],
+                              L["W_down"])
+    H.normwise_close(H.cpu(f["out"]).float().numpy(), want, H.OUT_TOL[dtype])
+
+
+def test_one_expert_layer_is_the_dense_swiglu_mlp():
+    """N = k = 1: the route is expert 0 with gate exactly 1 (a softmax over one logit), and the
+    layer is the dense SwiGLU MLP, checked here against fp64 matrix products directly."""
+    cfg = SMALL["fp32_one_expert"]
+    L = synth.make_layer(cfg, seed=6)
+    Ld = H.to_dev(L)
+    g = H.gpu_predict(cfg, Ld)
+    assert np.all(H.cpu(g["idx"]).numpy() == 0)
+    assert np.all(H.cpu(g["gates"]).numpy() == 1.0)
+    f = H.gpu_forward(cfg, Ld, g["idx"], g["gates"])
+    assert f["code"] == 0 and int(H.cpu(f["counts"])[0]) == cfg.T
+    x = L["x"].double()
+    a = x @ L["W_gate"][0].double().T
+    u = x @ L["W_up"][0].double().T
+    want = (a * torch.sigmoid(a) * u) @ L["W_down"][0].double().T
+    H.normwise_close(H.cpu(f["out"]).double().numpy(), want.numpy(), H.OUT_TOL["fp32"])
 
 
 def test_near_tie_counter_tracks_the_oracle_margin():
