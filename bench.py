@@ -330,6 +330,58 @@ def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
                                       *sh, o1, workspace=wsl), "pr2_moe_forward")
     ms = timed(pr3)
     out["pr3_step"] = dict(ms=ms, tokens_per_s=cfg.T / (ms * 1e-3), passes=3, T=cfg.T)
+    del wsl
+
+    # Training replay over long sequences (8 x 4096 = 32768 tokens) with recorded routes drawn
+    # Zipf(1.2) over the experts (per-expert rows 279 ... 31034): the same layer weights, new
+    # token rows; the routing call and the layer forward each timed alone.  At this size the
+    # routing kernel is no longer launch-bound and the expert GEMMs are compute-bound.
+    lcfg = synth.CONFIGS["qwen3_long_replay"]
+    if (cfg.d, cfg.N, cfg.k, cfg.m, cfg.dtype) == (lcfg.d, lcfg.N, lcfg.k, lcfg.m, lcfg.dtype):
+        Tl = lcfg.T
+        ldm = B.dims(Tl, cfg.d, cfg.N, cfg.k, cfg.m, cfg.n_shared, cfg.dtype)
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(7)
+        xl = torch.randn(Tl, cfg.d, generator=gen, device=dev).to(cfg.torch_dtype)
+        il = synth.make_zipf_routes(Tl, cfg.N, cfg.k, lcfg.zipf_s).to(dev)
+        gl = torch.empty(Tl, cfg.k, dtype=torch.float32, device=dev)
+        ol = torch.empty(Tl, cfg.d, dtype=cfg.torch_dtype, device=dev)
+        wl = B.alloc_workspace(ldm)
+
+        def route_l():
+            B.check(B.pr2_route_replay(ldm, xl, W2, il, gl, None, status), "pr2_route_replay")
+
+        def forward_l(evs=None):
+            B.check(B.pr2_moe_forward(ldm, xl, il, gl, L["W_gate"], L["W_up"], L["W_down"],
+                                      L["Ws_gate"], L["Ws_up"], L["Ws_down"], ol, workspace=wl,
+                                      status=status, events=evs), "pr2_moe_forward")
+        route_l()
+        ms_r = timed(route_l)
+        report("long_replay_route", ms_r,
+               cost.route_replay_work(Tl, cfg.d, cfg.N, cfg.k, cfg.dtype, False), T=Tl)
+        # the forward with an event at every stage boundary: the grouped GEMM launch alone too
+        sets = []
+        for i in range(iters + 3):
+            flush.fill_(i & 0xFF)
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+            for x in e:
+                x.record()
+            forward_l(B.stage_events(e))
+            sets.append(e)
+        torch.cuda.synchronize()
+        ms_f = statistics.median(e[0].elapsed_time(e[4]) for e in sets[3:])
+        ms_g = statistics.median(e[1].elapsed_time(e[3]) for e in sets[3:])
+        Fl = Tl * cfg.k
+        gw = cost.expert_mlp_work(Fl, cfg.d, cfg.m, cfg.N, cfg.dtype, a_rows=Tl)
+        fw = [cost.dispatch_work(Tl, cfg.d, cfg.k, cfg.dtype, gather=False), gw,
+              cost.combine_work(Tl, cfg.d, cfg.k, cfg.n_shared, cfg.dtype)]
+        report("long_replay_expert_gemm", ms_g, gw, T=Tl,
+               tensor_frac_sustained=gw.flops / (ms_g * 1e-3) / 1e12 / pk["bf16_sustained"],
+               routes="Zipf(1.2) over experts, seed 2; token rows N(0,1), seed 7")
+        report("long_replay_forward", ms_f, cost.KernelWork(sum(w.bytes for w in fw),
+                                                           sum(w.flops for w in fw)),
+               T=Tl, tokens_per_s=Tl / ((ms_r + ms_f) * 1e-3))
+        del wl, xl, ol
     if int(status.item()) != 0:
         raise RuntimeError(f"device status {int(status.item())} in the extra rows")
     return out
