@@ -167,7 +167,9 @@ pr2_status route_common(const pr2_dims* dims, bool predict, const void* h, const
     const int num_sms = num_sms_of_current_device();
     if (num_sms <= 0) return PR2_ERR_CUDA;
     const int mode = predict ? kModePredict : kModeReplay;
-    const int split = route_split(static_cast<int>(dm.T), dm.N, dm.d, mode, num_sms);
+    const bool compact = route_compact(static_cast<int>(dm.T), dm.N, mode, num_sms);
+    const int split =
+        compact ? 1 : route_split(static_cast<int>(dm.T), dm.N, dm.d, mode, num_sms);
     CUtensorMap tm_h, tm_w, tm_wp;
     if (!make_tmap_bf16(&tm_h, h, dm.d, dm.T, 64, kTileM) ||
         !make_tmap_bf16(&tm_w, W, dm.d, dm.N, 64, dm.N))
@@ -189,6 +191,7 @@ pr2_status route_common(const pr2_dims* dims, bool predict, const void* h, const
     a.near_tie = near_tie;
     a.status = status_dev;
     a.norm = (dm.flags & PR2_F_NORMALIZE_TOPK) ? 1 : 0;
+    a.compact = compact ? 1 : 0;
     err = launch_route_tc(mode, tm_h, tm_w, tm_wp, a, split, st);
   }
   return finish(err, dm.flags, status_dev, st);

@@ -72,6 +72,7 @@ struct RouteTcArgs {
   int64_t* near_tie;
   int32_t* status;
   int norm;                // PR2_F_NORMALIZE_TOPK: gates divided by their sum over the route
+  int compact;             // 1: half the pipeline stages, so two CTAs share an SM (split 1)
   // kModeLoss only (h = h_old, W = W_p)
   const float* p_old;      // [T, N] cached router logits
   const float* rho;        // [T_rho, N] teacher probabilities
@@ -84,6 +85,10 @@ struct RouteTcArgs {
 };
 // CTAs of the cluster that splits K for one 128-token tile (1 = no split).
 int route_split(int T, int N, int d, int mode, int num_sms);
+// Whether a launch over T tokens runs two CTAs per SM, each with half the pipeline stages and
+// no K split: when the 128-token tiles outnumber the SMs, so that one CTA's loads and finishing
+// overlap the other's MMAs instead of the tiles running as a second wave.
+bool route_compact(int T, int N, int mode, int num_sms);
 cudaError_t launch_route_tc(int mode, const CUtensorMap& tm_h, const CUtensorMap& tm_w,
                             const CUtensorMap& tm_wp, const RouteTcArgs& a, int split,
                             cudaStream_t st);

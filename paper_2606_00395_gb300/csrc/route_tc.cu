@@ -11,7 +11,9 @@
 // tcgen05.mma costs the same issue time for any N <= 256 (one M=128 x N x K=16 step), so a lone
 // tile's chain of d/16 MMAs, not bandwidth, bounds it, and only a K split shortens that chain:
 // CTA r multiplies K blocks [r KB/S, (r+1) KB/S) into a partial [128 x NB] fp32 accumulator
-// (NB = 2N columns [p_old | b] for predict, N for replay).
+// (NB = 2N columns [p_old | b] for predict, N for replay).  When the tiles outnumber the SMs
+// (S = 1), each CTA takes half the pipeline stages so that two run on an SM side by side, one
+// CTA's loads and finishing overlapping the other's MMAs (RouteTcArgs::compact).
 //
 // Warp roles: warp 0 = TMA producer, warp 1 = TMEM owner and MMA issuer, warps 2..5 = epilogue.
 // With S > 1 the partials are reduce-scattered by rows through distributed shared memory: CTA q
@@ -41,6 +43,8 @@ constexpr int kATileBytes = kTileM * kBK * 2;    // 16 KB
 constexpr int kKeep = kMaxTopK + 1;              // top-(k+1) kept for the margin
 constexpr int kMaxSplit = 8;
 constexpr int kMaxStages = 12;
+constexpr int kStageBudget = 192 * 1024;    // pipeline stages of a CTA alone on its SM
+constexpr int kCompactBudget = 96 * 1024;   // two CTAs per SM (more token tiles than SMs)
 
 struct RouteSmemLayout {
   int stages;
@@ -50,11 +54,11 @@ struct RouteSmemLayout {
   int total;         // dynamic smem bytes requested (incl. 1 KB alignment slack)
 };
 
-__host__ __device__ inline RouteSmemLayout route_layout(int N, bool predict) {
+__host__ __device__ inline RouteSmemLayout route_layout(int N, bool predict, bool compact) {
   RouteSmemLayout L;
   L.b_rows = predict ? 2 * N : N;
   L.stage_bytes = kATileBytes + L.b_rows * kBK * 2;
-  L.stages = (192 * 1024) / L.stage_bytes;
+  L.stages = (compact ? kCompactBudget : kStageBudget) / L.stage_bytes;
   if (L.stages > kMaxStages) L.stages = kMaxStages;
   if (L.stages < 2) L.stages = 2;
   L.bar_offset = L.stages * L.stage_bytes;
@@ -165,7 +169,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr bool loss = kMode == kModeLoss;
   extern __shared__ __align__(16) uint8_t smem_raw[];
   const int N = a.N, k = a.k;
-  const RouteSmemLayout L = route_layout(N, predict);
+  const RouteSmemLayout L = route_layout(N, predict, a.compact != 0);
   // 1024-B aligned base, kept as an offset into the shared array so the compiler knows every
   // derived pointer is shared memory.
   const uint32_t pad = (1024u - (smem_u32(smem_raw) & 1023u)) & 1023u;
@@ -616,9 +620,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 template <int kMode, int kSplit>
 cudaError_t set_smem_attr(int N) {
+  const cudaError_t err = cudaFuncSetAttribute(route_tc_kernel<kMode, kSplit>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               route_layout(N, kMode == kModePredict, false).total);
+  if (err != cudaSuccess) return err;
+  // all of the SM's unified L1 / shared storage as shared memory, so that two compact CTAs fit
   return cudaFuncSetAttribute(route_tc_kernel<kMode, kSplit>,
-                              cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              route_layout(N, kMode == kModePredict).total);
+                              cudaFuncAttributePreferredSharedMemoryCarveout,
+                              cudaSharedmemCarveoutMaxShared);
 }
 
 template <int kMode, int kSplit>
@@ -627,7 +636,7 @@ cudaError_t launch_split(const CUtensorMap& tm_h, const CUtensorMap& tm_w,
                          cudaStream_t st, int* max_clusters) {
   cudaError_t err = set_smem_attr<kMode, kSplit>(a.N);
   if (err != cudaSuccess) return err;
-  const size_t smem = route_layout(a.N, kMode == kModePredict).total;
+  const size_t smem = route_layout(a.N, kMode == kModePredict, a.compact != 0).total;
   if (max_clusters != nullptr) {  // occupancy query only
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(tiles * kSplit);
@@ -673,11 +682,40 @@ cudaError_t launch_any(int mode, const CUtensorMap& tm_h, const CUtensorMap& tm_
   }
 }
 
+// CTAs of route_tc_kernel<mode, 1> with the compact layout that fit on one SM by its shared
+// memory, registers and threads (0 on error).  Counted from the kernel's attributes and the
+// device limits: the occupancy query answers 1 for this kernel although two CTAs do run on
+// one SM side by side (a per-CTA %smid / %globaltimer record of a T = 32768 launch).
+template <int kMode>
+int compact_blocks_per_sm(int N) {
+  if (set_smem_attr<kMode, 1>(N) != cudaSuccess) return 0;
+  cudaFuncAttributes fa{};
+  if (cudaFuncGetAttributes(&fa, route_tc_kernel<kMode, 1>) != cudaSuccess) return 0;
+  int dev = 0, smem_sm = 0, reserved = 0, regs_sm = 0, threads_sm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) !=
+          cudaSuccess ||
+      cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev) !=
+          cudaSuccess ||
+      cudaDeviceGetAttribute(&regs_sm, cudaDevAttrMaxRegistersPerMultiprocessor, dev) !=
+          cudaSuccess ||
+      cudaDeviceGetAttribute(&threads_sm, cudaDevAttrMaxThreadsPerMultiProcessor, dev) !=
+          cudaSuccess)
+    return 0;
+  const size_t smem = route_layout(N, kMode == kModePredict, true).total + fa.sharedSizeBytes +
+                      static_cast<size_t>(reserved);
+  const int regs = ((fa.numRegs + 7) / 8) * 8 * kThreads;  // allocated per warp in 256s
+  int n = static_cast<int>(static_cast<size_t>(smem_sm) / smem);
+  if (regs > 0 && regs_sm / regs < n) n = regs_sm / regs;
+  if (threads_sm / kThreads < n) n = threads_sm / kThreads;
+  return n;
+}
+
 // Clusters of `split` CTAs of this kernel that can be resident at once (0 on error), cached
 // per device and shape.
-int max_active_clusters(int mode, int split, int N) {
+int max_active_clusters(int mode, int split, int N, bool compact = false) {
   struct Entry {
-    int dev, mode, split, N, clusters;
+    int dev, mode, split, N, compact, clusters;
   };
   static std::mutex mu;
   static Entry cache[64];
@@ -687,25 +725,43 @@ int max_active_clusters(int mode, int split, int N) {
   std::lock_guard<std::mutex> lock(mu);
   for (int i = 0; i < used; ++i)
     if (cache[i].dev == dev && cache[i].mode == mode && cache[i].split == split &&
-        cache[i].N == N)
+        cache[i].N == N && cache[i].compact == static_cast<int>(compact))
       return cache[i].clusters;
-  RouteTcArgs probe{};
-  probe.N = N;
-  CUtensorMap none{};
   int clusters = 0;
-  const cudaError_t err = launch_any(mode, none, none, none, probe, split, 1, nullptr, &clusters);
-  if (err != cudaSuccess) {
+  if (compact) {  // clusters of one CTA: CTAs per SM, times the SMs
+    const int per_sm = mode == kModePredict ? compact_blocks_per_sm<kModePredict>(N)
+                                            : compact_blocks_per_sm<kModeReplay>(N);
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
+      clusters = per_sm * sms;
     (void)cudaGetLastError();
-    clusters = 0;
+  } else {
+    RouteTcArgs probe{};
+    probe.N = N;
+    CUtensorMap none{};
+    const cudaError_t err =
+        launch_any(mode, none, none, none, probe, split, 1, nullptr, &clusters);
+    if (err != cudaSuccess) {
+      (void)cudaGetLastError();
+      clusters = 0;
+    }
   }
-  if (used < 64) cache[used++] = Entry{dev, mode, split, N, clusters};
+  if (used < 64) cache[used++] = Entry{dev, mode, split, N, static_cast<int>(compact), clusters};
   return clusters;
 }
 
 }  // namespace
 
+bool route_compact(int T, int N, int mode, int num_sms) {
+  const int tiles = (T + kTileM - 1) / kTileM;
+  if (tiles <= num_sms) return false;
+  const RouteSmemLayout L = route_layout(N, mode == kModePredict, true);
+  if (L.stages * L.stage_bytes > kCompactBudget) return false;  // not even two stages fit
+  return max_active_clusters(mode, 1, N, true) >= 2 * num_sms;
+}
+
 int route_split(int T, int N, int d, int mode, int num_sms) {
-  const RouteSmemLayout L = route_layout(N, mode == kModePredict);
+  const RouteSmemLayout L = route_layout(N, mode == kModePredict, false);
   const int tiles = (T + kTileM - 1) / kTileM;
   const int KB = d / kBK;
   if (route_recv_bytes(L.b_rows) > L.stages * L.stage_bytes) return 1;
@@ -722,7 +778,7 @@ cudaError_t launch_route_tc(int mode, const CUtensorMap& tm_h, const CUtensorMap
                             cudaStream_t st) {
   if (a.T == 0) return cudaSuccess;
   if (split < 1 || split > kMaxSplit || a.N % split != 0 || (a.N / split) % 16 != 0 ||
-      (a.d / kBK) % split != 0)
+      (a.d / kBK) % split != 0 || (a.compact != 0 && split != 1))
     return cudaErrorInvalidValue;
   const int tiles = (a.T + kTileM - 1) / kTileM;
   return launch_any(mode, tm_h, tm_w, tm_wp, a, split, tiles, st, nullptr);

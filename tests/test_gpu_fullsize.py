@@ -109,6 +109,24 @@ def test_long_replay_with_zipf_routes():
     print(f"zipf counts {counts.min()}..{counts.max()}, output error {err:.2e}")
 
 
+def test_long_batch_routing_both_modes():
+    """T = 32768 tokens: 256 token tiles, more than the GPU has SMs, so routing runs two CTAs
+    per SM with half the pipeline stages each; routes and gates on a token sample in both
+    modes, the replay probabilities too."""
+    cfg = synth.CONFIGS["qwen3_long_replay"]
+    L = synth.make_layer(cfg, device="cuda")
+    g = H.gpu_predict(cfg, L)
+    sample = synth.make_token_sample(cfg.T, 384, 6).numpy()
+    exempt, n, orc = _routing_check(cfg, L, g, sample=sample)
+    W2 = synth.make_drifted_router(L["W_router"])
+    r = H.gpu_replay(cfg, L, W2, g["idx"])
+    orep = oracle.route_replay(H.cpu(L["x"])[sample], H.cpu(W2), H.cpu(g["idx"]).numpy()[sample])
+    H.rowwise_close(H.cpu(r["gates"]).numpy()[sample], orep["gates"])
+    H.rowwise_close(H.cpu(r["probs"]).numpy()[sample], orep["probs"])
+    assert int(g["status"].item()) == 0 and int(r["status"].item()) == 0
+    print(f"long batch routing: {exempt}/{n} near ties (sampled)")
+
+
 def test_deepseek_v3_layer_with_shared_expert():
     cfg = synth.CONFIGS["deepseek_v3"]
     L = synth.make_layer(cfg, device="cuda")
