@@ -76,6 +76,11 @@ __host__ __device__ inline uint32_t tmem_cols_for(int cols) {
   return c;
 }
 
+// Barrier over `count` threads (whole warps) on hardware barrier `id` (0 is __syncthreads).
+__device__ __forceinline__ void named_bar_sync(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 // Compare-exchange leaving the larger key in a.
 __device__ __forceinline__ void cas_desc(uint64_t& a, uint64_t& b) {
   const bool sw = b > a;
@@ -352,8 +357,28 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     cluster_sync();  // every partial row has landed
+    if (epi) {
+      // Sum the S received copies of this CTA's rows once, in source order, into source 0's
+      // slots: consecutive threads take consecutive 16-byte words (no bank conflicts), so the
+      // finishing threads then read one value per column instead of S strided ones.
+      float4* red = reinterpret_cast<float4*>(smem);
+      const int n4 = nb4 * R;  // 16-byte words of one source
+      for (int i = threadIdx.x - 64; i < n4; i += 128) {
+        float4 v = red[i];
+#pragma unroll
+        for (int src = 1; src < split; ++src) {
+          const float4 w = red[src * n4 + i];
+          v.x += w.x;
+          v.y += w.y;
+          v.z += w.z;
+          v.w += w.w;
+        }
+        red[i] = v;
+      }
+      named_bar_sync(1, 128);  // the four epilogue warps
+    }
   }
-  // Columns [c, c + 16) of the finished row: summed partials (S > 1) or TMEM (S = 1).
+  // Columns [c, c + 16) of the finished row: the summed partials (S > 1) or TMEM (S = 1).
   auto load16 = [&](int c, uint32_t (&r)[16]) {
     if (split == 1) {
       tmem_ld16(trow + c, r);
@@ -362,15 +387,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      float4 v = recv[(c / 4 + j) * R + lr];
-#pragma unroll
-      for (int src = 1; src < split; ++src) {
-        const float4 w = recv[(src * nb4 + c / 4 + j) * R + lr];
-        v.x += w.x;
-        v.y += w.y;
-        v.z += w.z;
-        v.w += w.w;
-      }
+      const float4 v = recv[(c / 4 + j) * R + lr];
       r[4 * j] = __float_as_uint(v.x);
       r[4 * j + 1] = __float_as_uint(v.y);
       r[4 * j + 2] = __float_as_uint(v.z);
