@@ -18,8 +18,13 @@ SMALL = {
     # fp32 SIMT path, the tiny workload exactly
     "tiny_fp32": synth.CONFIGS["tiny_fp32"],
     # fp32 with N = 6 experts: dispatch takes its three-kernel path (the fused cooperative
-    # dispatch needs N % 4 == 0)
+    # dispatch needs N % 4 == 0), with one and with 36 blocks of slots
     "fp32_n6": synth.LayerConfig("fp32_n6", T=300, d=64, N=6, k=3, m=96, dtype="fp32"),
+    "fp32_n6_wide": synth.LayerConfig("fp32_n6_wide", T=3000, d=64, N=6, k=3, m=96,
+                                      dtype="fp32"),
+    # bf16, 9600 slots over 38 blocks of the fused cooperative dispatch, N = 32, m = 64
+    "bf16_fused_dispatch": synth.LayerConfig("bf16_fused_dispatch", T=1200, d=128, N=32, k=8,
+                                             m=64),
     # bf16, ~175 rows per expert -> 2 M-tiles per expert, 2 gate/up N-tiles, ragged T
     "bf16_multitile": synth.LayerConfig("bf16_multitile", T=700, d=256, N=16, k=4, m=256),
     # bf16, partial N-tiles in both GEMMs (m = 192 = 128 + 64, d = 320 = 256 + 64), k = 6
