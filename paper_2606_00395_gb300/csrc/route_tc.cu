@@ -18,8 +18,9 @@
 // Warp roles: warp 0 = TMA producer, warp 1 = TMEM owner and MMA issuer, warps 2..5 = epilogue.
 // With S > 1 the partials are reduce-scattered by rows through distributed shared memory: CTA q
 // receives rows [q 128/S, (q+1) 128/S) of every CTA's partial, stored [source][column/4][row][4]
-// so that each warp store moves contiguous bytes, and sums them in source order (deterministic).
-// Each row is then finished by S consecutive threads, thread `part` owning experts
+// so that each warp store moves contiguous bytes; the four epilogue warps then sum the S copies
+// once, in source order (deterministic), walking consecutive 16-byte words so that no two lanes
+// of a warp hit one bank.  Each row is then finished by S consecutive threads, thread `part` owning experts
 // [part N/S, (part+1) N/S); with S = 1 one thread finishes its row straight from TMEM.  A thread
 // reduces its experts to a max, a sum of exp(z - max) and (predict) its top-16 by 64-bit keys
 // (orderable z bits, inverted expert index: z descending, ties to the lower expert), built by
