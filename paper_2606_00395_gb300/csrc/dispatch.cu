@@ -93,6 +93,45 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* sh, int* total) 
   return incl - v;
 }
 
+// The grouped GEMM's M-tile table (entry i belongs to the expert whose tile range contains i;
+// its per-M-tile readiness counter is cleared) and the static tile tables of the shared experts
+// (every token: gate/up reads rows of h, down rows of Hs), from the experts' row offsets ex_off
+// and first tiles ex_tile (N + 1 entries each, in shared memory); num_tiles[0..1] = their
+// lengths.  Called by every thread of one block.
+__device__ void write_tile_tables(int N, int64_t T, int n_shared, const int* ex_off,
+                                  const int* ex_tile, TileEntry* __restrict__ tiles,
+                                  int32_t* __restrict__ num_tiles,
+                                  TileEntry* __restrict__ stiles1,
+                                  TileEntry* __restrict__ stiles2, int32_t* __restrict__ ready) {
+  const int tid = threadIdx.x;
+  const int all_tiles = ex_tile[N];
+  const int mt_T = static_cast<int>((T + kTileM - 1) / kTileM);
+  if (tid == 0) {
+    num_tiles[0] = all_tiles;
+    num_tiles[1] = n_shared * mt_T;
+  }
+  for (int i = tid; i < all_tiles; i += blockDim.x) {
+    int lo = 0, hi = N - 1;
+    while (lo < hi) {  // last expert with ex_tile[ex] <= i
+      const int mid = (lo + hi + 1) >> 1;
+      if (ex_tile[mid] <= i) lo = mid; else hi = mid - 1;
+    }
+    const int j = i - ex_tile[lo];
+    const int r0 = ex_off[lo] + j * kTileM;
+    const int left = ex_off[lo + 1] - r0;
+    tiles[i] = TileEntry{lo, r0, left < kTileM ? left : kTileM, r0};
+    if (ready != nullptr) ready[i] = 0;  // per M-tile counter of the fused expert GEMM
+  }
+  for (int i = tid; i < n_shared * mt_T; i += blockDim.x) {
+    const int j = i / mt_T, m = i - j * mt_T;
+    const int r0 = m * kTileM;
+    const int rows = (T - r0) < kTileM ? static_cast<int>(T - r0) : kTileM;
+    const int o0 = static_cast<int>(j * T) + r0;
+    stiles1[i] = TileEntry{j, r0, rows, o0};
+    stiles2[i] = TileEntry{j, o0, rows, o0};
+  }
+}
+
 // One block of 1024 threads = G groups of N_pad threads: thread (g, e) owns expert e over the
 // block range of group g, so the per-expert scans over blocks run G-way parallel.
 __global__ void __launch_bounds__(1024)
@@ -150,7 +189,6 @@ __global__ void __launch_bounds__(1024)
   }
   if (tid == 0) {
     offsets[N] = all_rows;
-    num_tiles[0] = all_tiles;
     ex_off[N] = all_rows;
     ex_tile[N] = all_tiles;
   }
@@ -170,30 +208,7 @@ __global__ void __launch_bounds__(1024)
       }
     }
   }
-  // M-tile table: entry i belongs to the expert whose tile range contains i
-  for (int i = tid; i < all_tiles; i += blockDim.x) {
-    int lo = 0, hi = N - 1;
-    while (lo < hi) {  // last expert with ex_tile[ex] <= i
-      const int mid = (lo + hi + 1) >> 1;
-      if (ex_tile[mid] <= i) lo = mid; else hi = mid - 1;
-    }
-    const int j = i - ex_tile[lo];
-    const int r0 = ex_off[lo] + j * kTileM;
-    const int left = ex_off[lo + 1] - r0;
-    tiles[i] = TileEntry{lo, r0, left < kTileM ? left : kTileM, r0};
-    if (ready != nullptr) ready[i] = 0;  // per M-tile counter of the fused expert GEMM
-  }
-  // Shared experts: every token, fixed tiles.  Gate/up reads h rows, down reads Hs rows.
-  const int mt_T = static_cast<int>((T + kTileM - 1) / kTileM);
-  for (int i = tid; i < n_shared * mt_T; i += blockDim.x) {
-    const int j = i / mt_T, m = i - j * mt_T;
-    const int r0 = m * kTileM;
-    const int rows = (T - r0) < kTileM ? static_cast<int>(T - r0) : kTileM;
-    const int o0 = static_cast<int>(j * T) + r0;
-    stiles1[i] = TileEntry{j, r0, rows, o0};
-    stiles2[i] = TileEntry{j, o0, rows, o0};
-  }
-  if (tid == 0) num_tiles[1] = n_shared * mt_T;
+  write_tile_tables(N, T, n_shared, ex_off, ex_tile, tiles, num_tiles, stiles1, stiles2, ready);
 }
 
 __global__ void __launch_bounds__(kDispatchChunk)
@@ -376,32 +391,9 @@ __global__ void __launch_bounds__(kDispatchChunk)
       counts[tid] = total;
       offsets[tid] = off;
     }
-    if (tid == 0) {
-      offsets[N] = all_rows;
-      num_tiles[0] = all_tiles;
-      num_tiles[1] = n_shared * static_cast<int>((T + kTileM - 1) / kTileM);
-    }
-    for (int i = tid; i < all_tiles; i += blockDim.x) {
-      int lo = 0, hi = N - 1;
-      while (lo < hi) {  // last expert with ex_tile[ex] <= i
-        const int mid = (lo + hi + 1) >> 1;
-        if (ex_tile[mid] <= i) lo = mid; else hi = mid - 1;
-      }
-      const int j = i - ex_tile[lo];
-      const int r0 = ex_off[lo] + j * kTileM;
-      const int left = ex_off[lo + 1] - r0;
-      tiles[i] = TileEntry{lo, r0, left < kTileM ? left : kTileM, r0};
-      if (ready != nullptr) ready[i] = 0;  // per M-tile counter of the fused expert GEMM
-    }
-    const int mt_T = static_cast<int>((T + kTileM - 1) / kTileM);
-    for (int i = tid; i < n_shared * mt_T; i += blockDim.x) {
-      const int j = i / mt_T, m = i - j * mt_T;
-      const int r0 = m * kTileM;
-      const int rows = (T - r0) < kTileM ? static_cast<int>(T - r0) : kTileM;
-      const int o0 = static_cast<int>(j * T) + r0;
-      stiles1[i] = TileEntry{j, r0, rows, o0};
-      stiles2[i] = TileEntry{j, o0, rows, o0};
-    }
+    if (tid == 0) offsets[N] = all_rows;
+    write_tile_tables(N, T, n_shared, ex_off, ex_tile, tiles, num_tiles, stiles1, stiles2,
+                      ready);
   }
   // ---- 3. stable placement: per-warp bases, then ranks within the warp
   for (int x = tid; x < N; x += blockDim.x) {
