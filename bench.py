@@ -19,6 +19,7 @@ import json
 import os
 import statistics
 import subprocess
+import tempfile
 import sys
 import time
 
@@ -94,7 +95,10 @@ class ClockSampler:
 
     def __init__(self, index: int):
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+        # raw samples: a scratch file (PR2_CLOCKS_DIR to keep them elsewhere); the JSON line
+        # carries the summary
+        self.path = os.path.join(os.environ.get("PR2_CLOCKS_DIR", tempfile.gettempdir()),
+                                 f"pr2_clocks_rank{index}_{os.getpid()}.csv")
         uuid = str(getattr(torch.cuda.get_device_properties(index), "uuid", index))
         sel = uuid if uuid.startswith("GPU-") else (f"GPU-{uuid}" if "-" in uuid else str(index))
         try:
@@ -117,7 +121,11 @@ class ClockSampler:
             self.proc.kill()
         self.fh.close()
         rows = []
-        for line in open(self.path):
+        with open(self.path) as fh:
+            lines = fh.readlines()
+        if "PR2_CLOCKS_DIR" not in os.environ:
+            os.remove(self.path)
+        for line in lines:
             parts = [x.strip() for x in line.split(",")]
             if len(parts) < 7:
                 continue
