@@ -775,6 +775,7 @@ bool route_compact(int T, int N, int mode, int num_sms) {
   if (tiles <= num_sms) return false;
   const RouteSmemLayout L = route_layout(N, mode == kModePredict, true);
   if (L.stages * L.stage_bytes > kCompactBudget) return false;  // not even two stages fit
+  if (2 * tmem_cols_for(L.b_rows) > 512) return false;           // two accumulators in TMEM
   return max_active_clusters(mode, 1, N, true) >= 2 * num_sms;
 }
 
