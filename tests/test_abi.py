@@ -202,3 +202,16 @@ def test_unknown_flags_are_rejected(lib):
     code = lib.pr2_route_predict(ctypes.byref(bad), fake, fake, fake, fake, fake, None, None, None,
                                  None)
     assert code == 1  # PR2_ERR_INVALID_ARG, before any launch
+
+
+def test_static_scratch_holds_up_to_743_tokens_of_the_qwen3_layer(lib):
+    """pr2_moe_forward_static's fixed scratch: the Qwen3-shaped layer fits up to 743 tokens (the
+    limit pr2.h states); one more token is rejected with PR2_ERR_WORKSPACE before any launch."""
+    scratch = B.pr2_static_scratch_bytes()
+    assert B.pr2_moe_workspace_bytes(B.dims(743, 2048, 128, 8, 768)) <= scratch
+    over = B.dims(744, 2048, 128, 8, 768)
+    assert B.pr2_moe_workspace_bytes(over) > scratch
+    fake = ctypes.c_void_p(256)
+    slib = B._static_lib()
+    assert slib.pr2_moe_forward_static(ctypes.byref(over), fake, fake, fake, fake, fake, fake,
+                                       None, None, None, fake, None, None, None, None) == 6
