@@ -75,6 +75,29 @@ def test_qwen3_layer_both_modes():
     print(f"qwen3 output error replay {err:.2e} rollout {err2:.2e}")
 
 
+def test_qwen3_shape_ragged_batch():
+    """The Qwen3-shaped layer with T = 4001 (the last token tile 33 rows): every route against
+    the oracle, counts and permutation bit-exact, layer outputs on a token sample."""
+    cfg = synth.CONFIGS["qwen3_30b_a3b"].scaled(4001)
+    L = synth.make_layer(cfg, device="cuda")
+    g = H.gpu_predict(cfg, L)
+    exempt, n, orc = _routing_check(cfg, L, g)
+    f = H.gpu_forward(cfg, L, g["idx"], g["gates"])
+    assert f["code"] == 0 and int(f["status"].item()) == 0
+    gidx = H.cpu(g["idx"]).numpy()
+    operm = oracle.permute(gidx, cfg.N)
+    assert np.array_equal(H.cpu(f["counts"]).numpy(), operm["counts"])
+    assert np.array_equal(H.cpu(f["perm"]).numpy(), operm["perm"])
+    toks = np.unique(np.concatenate([synth.make_token_sample(cfg.T, 40, 7).numpy(),
+                                     np.arange(cfg.T - 8, cfg.T)]))  # + the ragged tile's end
+    idx_s = gidx[toks]
+    Wg, Wu, Wd, idx_c = H.compact_experts(L, idx_s)
+    want = oracle.moe_forward(H.cpu(L["x"])[toks], idx_c, H.cpu(g["gates"]).numpy()[toks],
+                              Wg, Wu, Wd)
+    err = H.normwise_close(H.cpu(f["out"]).float().numpy()[toks], want, H.OUT_TOL[cfg.dtype])
+    print(f"qwen3 T=4001: {exempt}/{n} near ties, output error {err:.2e}")
+
+
 def test_qwen3_decode_batch_rollout():
     cfg = synth.CONFIGS["qwen3_decode"]
     L = synth.make_layer(cfg, device="cuda")
@@ -109,11 +132,12 @@ def test_long_replay_with_zipf_routes():
     print(f"zipf counts {counts.min()}..{counts.max()}, output error {err:.2e}")
 
 
-def test_long_batch_routing_both_modes():
-    """T = 32768 tokens: 256 token tiles, more than the GPU has SMs, so routing runs two CTAs
-    per SM with half the pipeline stages each; routes and gates on a token sample in both
-    modes, the replay probabilities too."""
-    cfg = synth.CONFIGS["qwen3_long_replay"]
+@pytest.mark.parametrize("T", [32768, 20001])
+def test_long_batch_routing_both_modes(T):
+    """T = 32768 (256 token tiles) and T = 20001 (157 tiles, the last one ragged): more tiles
+    than the GPU has SMs, so routing runs two CTAs per SM with half the pipeline stages each;
+    routes and gates on a token sample in both modes, the replay probabilities too."""
+    cfg = synth.CONFIGS["qwen3_long_replay"].scaled(T)
     L = synth.make_layer(cfg, device="cuda")
     g = H.gpu_predict(cfg, L)
     sample = synth.make_token_sample(cfg.T, 384, 6).numpy()
