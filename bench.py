@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--extras-iters", type=int, default=50,
                     help="timed calls of each widening row (after 3 untimed)")
+    ap.add_argument("--no-deepseek", action="store_true",
+                    help="skip the DeepSeek-V3-shaped layer among the extras")
     return ap.parse_args()
 
 
@@ -181,6 +183,20 @@ def host_layer(cfg, L):
 
 # ----------------------------------------------------------------------------------- pr2 arm
 
+def kernel_roofline(w, ms, pk, tc_peak):
+    """Roofline of one kernel from its algorithmic work `w` and mean duration `ms`: the bound
+    that allows the longer time (tensor at `tc_peak` or HBM), and measured time over it."""
+    t_hbm = w.bytes / (pk["hbm"] * 1e9) * 1e3
+    t_tc = w.flops / (tc_peak * 1e12) * 1e3
+    if t_tc > t_hbm:
+        return dict(ms=ms, bound="tensor", achieved=w.flops / (ms * 1e-3) / 1e12, peak=tc_peak,
+                    unit="TFLOP/s", frac=t_tc / ms, algorithmic_flops=w.flops,
+                    algorithmic_bytes=w.bytes)
+    return dict(ms=ms, bound="hbm", achieved=w.bytes / (ms * 1e-3) / 1e9, peak=pk["hbm"],
+                unit="GB/s", frac=t_hbm / ms, algorithmic_flops=w.flops,
+                algorithmic_bytes=w.bytes)
+
+
 def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
     """The rows that widen the hot path, each timed alone on the device (CUDA events around the
     call, L2 flushed before every call, median of ``iters``) against its own roofline:
@@ -287,9 +303,8 @@ def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
     graph_ms = timed(graph.replay, pre=lambda: hd.copy_(h0))
     per_layer = [cost.route_predict_work(Td, cfg.d, cfg.N, cfg.k, cfg.dtype, True),
                  cost.dispatch_work(Td, cfg.d, cfg.k, cfg.dtype, gather=cfg.dtype == "fp32"),
-                 cost.expert_gate_up_work(Td * cfg.k, cfg.d, cfg.m, cfg.N, cfg.dtype,
-                                          a_rows=Td if cfg.dtype == "bf16" else None),
-                 cost.expert_down_work(Td * cfg.k, cfg.d, cfg.m, cfg.N, cfg.dtype),
+                 cost.expert_mlp_algorithmic_work(Td * cfg.k, cfg.d, cfg.m, cfg.N, cfg.dtype,
+                                                  a_rows=0),  # h counted by routing
                  cost.combine_work(Td, cfg.d, cfg.k, cfg.n_shared, cfg.dtype)]
     work = cost.KernelWork(Ld * sum(w.bytes for w in per_layer),
                            Ld * sum(w.flops for w in per_layer))
@@ -380,7 +395,7 @@ def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
         ms_f = statistics.median(e[0].elapsed_time(e[4]) for e in sets[3:])
         ms_g = statistics.median(e[1].elapsed_time(e[3]) for e in sets[3:])
         Fl = Tl * cfg.k
-        gw = cost.expert_mlp_work(Fl, cfg.d, cfg.m, cfg.N, cfg.dtype, a_rows=Tl)
+        gw = cost.expert_mlp_algorithmic_work(Fl, cfg.d, cfg.m, cfg.N, cfg.dtype, a_rows=Tl)
         fw = [cost.dispatch_work(Tl, cfg.d, cfg.k, cfg.dtype, gather=False), gw,
               cost.combine_work(Tl, cfg.d, cfg.k, cfg.n_shared, cfg.dtype)]
         report("long_replay_expert_gemm", ms_g, gw, T=Tl,
@@ -392,6 +407,107 @@ def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
         del wl, xl, ol
     if int(status.item()) != 0:
         raise RuntimeError(f"device status {int(status.item())} in the extra rows")
+    return out
+
+
+def measure_layer_modes(cfg, flush, pk, iters, seed=0):
+    """Both modes of one MoE layer workload timed on the device (the bench step's calls, CUDA
+    events at the mode boundaries, L2 flushed before every step, median of ``iters`` after 3
+    untimed), then a pass with an event at every stage boundary for the per-kernel split, each
+    kernel against its roofline: routing against the tensor bound where its 4TdN FLOPs outlast
+    its bytes (the DeepSeek-V3 shape), the routed + shared expert GEMMs against the larger of
+    the tensor time and the weight stream."""
+    dev = "cuda"
+    L = synth.make_layer(cfg, seed=seed, device=dev)
+    W2 = synth.make_drifted_router(L["W_router"], seed=seed)
+    dm = B.dims(cfg.T, cfg.d, cfg.N, cfg.k, cfg.m, cfg.n_shared, cfg.dtype)
+    ws = B.alloc_workspace(dm)
+    idx, gates, logits = B.alloc_route(dm, logits=True)
+    rg = torch.empty_like(gates)
+    o1 = torch.empty(cfg.T, cfg.d, dtype=cfg.torch_dtype, device=dev)
+    o2 = torch.empty_like(o1)
+    counts = torch.empty(cfg.N, dtype=torch.int32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    sh = (L["Ws_gate"], L["Ws_up"], L["Ws_down"])
+
+    def ev():
+        e = torch.cuda.Event(enable_timing=True)
+        e.record()
+        return e
+
+    def one(marks, st1=None, st2=None):
+        marks[0].record()
+        B.check(B.pr2_route_predict(dm, L["x"], L["W_router"], L["W_pred"], idx, gates, logits,
+                                    None, status), "pr2_route_predict")
+        if len(marks) > 3:
+            marks[3].record()
+        B.check(B.pr2_moe_forward(dm, L["x"], idx, gates, L["W_gate"], L["W_up"], L["W_down"],
+                                  *sh, o1, counts=counts, workspace=ws, status=status,
+                                  events=st1), "pr2_moe_forward")
+        marks[1].record()
+        B.check(B.pr2_route_replay(dm, L["x"], W2, idx, rg, None, status), "pr2_route_replay")
+        if len(marks) > 3:
+            marks[4].record()
+        B.check(B.pr2_moe_forward(dm, L["x"], idx, rg, L["W_gate"], L["W_up"], L["W_down"],
+                                  *sh, o2, workspace=ws, status=status, events=st2),
+                "pr2_moe_forward")
+        marks[2].record()
+
+    sets = []
+    for i in range(iters + 3):
+        flush.fill_(i & 0xFF)
+        m = [ev() for _ in range(3)]
+        one(m)
+        sets.append(m)
+    torch.cuda.synchronize()
+    roll = statistics.median(m[0].elapsed_time(m[1]) for m in sets[3:])
+    rep = statistics.median(m[1].elapsed_time(m[2]) for m in sets[3:])
+    step = statistics.median(m[0].elapsed_time(m[2]) for m in sets[3:])
+    # per-kernel pass: stage events inside both forwards
+    per = dict(route_predict=[], route_replay=[], dispatch=[], expert_gemm=[], combine=[])
+    for i in range(iters + 3):
+        flush.fill_(i & 0xFF)
+        m = [ev() for _ in range(5)]
+        a = [ev() for _ in range(5)]
+        b = [ev() for _ in range(5)]
+        one(m, B.stage_events(a), B.stage_events(b))
+        torch.cuda.synchronize()
+        if i < 3:
+            continue
+        per["route_predict"].append(m[0].elapsed_time(m[3]))
+        per["route_replay"].append(m[1].elapsed_time(m[4]))
+        for st in (a, b):
+            per["dispatch"].append(st[0].elapsed_time(st[1]))
+            per["expert_gemm"].append(st[1].elapsed_time(st[3]))
+            per["combine"].append(st[3].elapsed_time(st[4]))
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())} in the {cfg.name} layer")
+    hit = int((counts > 0).sum().item())
+    F = cfg.T * cfg.k
+    gw = cost.expert_mlp_algorithmic_work(F, cfg.d, cfg.m, hit, cfg.dtype, a_rows=cfg.T)
+    if cfg.n_shared:
+        sw = cost.expert_mlp_algorithmic_work(cfg.T * cfg.n_shared, cfg.d, cfg.m, cfg.n_shared,
+                                              cfg.dtype, a_rows=0)
+        gw = cost.KernelWork(gw.bytes + sw.bytes, gw.flops + sw.flops)
+    work = dict(route_predict=cost.route_predict_work(cfg.T, cfg.d, cfg.N, cfg.k, cfg.dtype,
+                                                      True),
+                route_replay=cost.route_replay_work(cfg.T, cfg.d, cfg.N, cfg.k, cfg.dtype),
+                dispatch=cost.dispatch_work(cfg.T, cfg.d, cfg.k, cfg.dtype),
+                expert_gemm=gw,
+                combine=cost.combine_work(cfg.T, cfg.d, cfg.k, cfg.n_shared, cfg.dtype))
+    kernels = {n: kernel_roofline(w, statistics.median(per[n]), pk, pk["bf16"])
+               for n, w in work.items()}
+    g = kernels["expert_gemm"]
+    g["tensor_frac"] = gw.flops / (pk["bf16"] * 1e12) / (g["ms"] * 1e-3)
+    out = dict(workload=cfg.name, T=cfg.T, d=cfg.d, N=cfg.N, k=cfg.k, m=cfg.m,
+               n_shared=cfg.n_shared, experts_hit=hit,
+               tokens_per_s=cfg.T / (step * 1e-3), ms_per_step=step,
+               rollout_tokens_per_s=cfg.T / (roll * 1e-3),
+               replay_tokens_per_s=cfg.T / (rep * 1e-3), kernels=kernels,
+               note="both modes as in the bench step; median of per-step device times, L2 "
+                    "flushed before every step")
+    del L, W2, ws
+    torch.cuda.empty_cache()
     return out
 
 
@@ -518,46 +634,59 @@ def run_pr2(args, rank, world, local_rank):
         "route_predict": cost.route_predict_work(cfg.T, cfg.d, cfg.N, cfg.k, cfg.dtype, True),
         "route_replay": cost.route_replay_work(cfg.T, cfg.d, cfg.N, cfg.k, cfg.dtype, False),
         "dispatch": cost.dispatch_work(cfg.T, cfg.d, cfg.k, cfg.dtype, gather=cfg.dtype == "fp32"),
-        "expert_gemm": cost.expert_mlp_work(F, cfg.d, cfg.m, hit, cfg.dtype,
-                                            a_rows=cfg.T if cfg.dtype == "bf16" else None),
+        # the fused minimum of the grouped GEMMs: h once and the hit experts' weights (the H
+        # round trip and the Y write of this design are counted in `modeled_bytes`)
+        "expert_gemm": cost.expert_mlp_algorithmic_work(
+            F, cfg.d, cfg.m, hit, cfg.dtype, a_rows=cfg.T),
         "combine": cost.combine_work(cfg.T, cfg.d, cfg.k, cfg.n_shared, cfg.dtype),
     }
+    modeled = cost.expert_mlp_work(F, cfg.d, cfg.m, hit, cfg.dtype,
+                                   a_rows=cfg.T if cfg.dtype == "bf16" else None).bytes
     if cfg.n_shared:
-        sw = cost.expert_mlp_work(cfg.T * cfg.n_shared, cfg.d, cfg.m, cfg.n_shared, cfg.dtype)
+        sw = cost.expert_mlp_algorithmic_work(cfg.T * cfg.n_shared, cfg.d, cfg.m, cfg.n_shared,
+                                              cfg.dtype, a_rows=0)
         work["expert_gemm"] = cost.KernelWork(work["expert_gemm"].bytes + sw.bytes,
                                               work["expert_gemm"].flops + sw.flops)
-    kernels = {}
-    for name, w in work.items():
-        ms = mean[name]
-        t_hbm = w.bytes / (pk["hbm"] * 1e9) * 1e3
-        t_tc = w.flops / (pk["bf16"] * 1e12) * 1e3
-        if t_tc > t_hbm:
-            kernels[name] = dict(ms=ms, bound="tensor", achieved=w.flops / (ms * 1e-3) / 1e12,
-                                 peak=pk["bf16"], unit="TFLOP/s", frac=t_tc / ms,
-                                 algorithmic_flops=w.flops, algorithmic_bytes=w.bytes)
-        else:
-            kernels[name] = dict(ms=ms, bound="hbm", achieved=w.bytes / (ms * 1e-3) / 1e9,
-                                 peak=pk["hbm"], unit="GB/s", frac=t_hbm / ms,
-                                 algorithmic_flops=w.flops, algorithmic_bytes=w.bytes)
+        modeled += cost.expert_mlp_work(cfg.T * cfg.n_shared, cfg.d, cfg.m, cfg.n_shared,
+                                        cfg.dtype).bytes
+    timed_s = total_ms / 1e3 / world
+    # The sustained bf16 peak (a GEMM looped for seconds under the power cap) applies only to a
+    # run whose clock record shows the power cap during a timed region of seconds; otherwise
+    # the burst peak (a GEMM timed alone at full clock) is the denominator.
+    sustained = bool(clk and "sw_power_cap" in clk.get("reasons", []) and timed_s >= 2.0)
+    tc_peak = pk["bf16_sustained"] if sustained else pk["bf16"]
+    kernels = {name: kernel_roofline(w, mean[name], pk, tc_peak) for name, w in work.items()}
     dom = "expert_gemm"
     dk = kernels[dom]
-    # The tensor-core fraction of the grouped GEMM, beside its binding (HBM) bound: against the
-    # burst bf16 peak (a GEMM timed alone) and the sustained one (a GEMM inside a long run of
-    # steps under the power cap, as here).
-    dk["tensor_frac"] = work[dom].flops / (pk["bf16"] * 1e12) * 1e3 / dk["ms"]
-    dk["tensor_frac_sustained"] = work[dom].flops / (pk["bf16_sustained"] * 1e12) * 1e3 / dk["ms"]
-    roofline = dict(kernel="expert_tc_kernel (routed gate/up + down, one launch)",
-                    bound=dk["bound"], achieved=dk["achieved"],
-                    peak=dk["peak"], unit=dk["unit"], frac=dk["frac"],
-                    traffic=measured_traffic(f"{cfg.name}/{dom}"),
-                    peak_source=f"{pk['source']} (MEASURED_PEAKS.json burst)"
-                    if pk["source"] == "measured" else "fallback",
-                    algorithmic=("flops" if dk["bound"] == "tensor" else "bytes"),
-                    tensor_frac=dk["tensor_frac"],
-                    tensor_frac_sustained=dk["tensor_frac_sustained"],
+    dk["modeled_bytes"] = modeled
+    # The grouped GEMM is the one dense contraction of the path: its roofline is the tensor
+    # pipe (FLOPs / duration against the bf16 peak); `combined_frac` is the time the tighter of
+    # its two bounds allows (tensor, or HBM on h + the experts' weights) over the duration.
+    w = work[dom]
+    traffic = measured_traffic(f"{cfg.name}/{dom}")
+    roofline = dict(kernel="expert_tc_kernel (routed gate/up + down, one launch)"
+                    + (" + shared-expert GEMMs" if cfg.n_shared else ""),
+                    bound="tensor", achieved=w.flops / (dk["ms"] * 1e-3) / 1e12,
+                    peak=tc_peak, unit="TFLOP/s",
+                    frac=w.flops / (tc_peak * 1e12) / (dk["ms"] * 1e-3),
+                    traffic=traffic,
+                    peak_source=(f"{pk['source']} (MEASURED_PEAKS.json "
+                                 f"{'sustained' if sustained else 'burst'})"
+                                 if pk["source"] == "measured" else "fallback"),
+                    algorithmic="flops",
+                    algorithmic_flops=w.flops, algorithmic_bytes=w.bytes,
+                    combined_frac=dk["frac"], combined_bound=dk["bound"],
+                    hbm_frac=w.bytes / (pk["hbm"] * 1e9) / (dk["ms"] * 1e-3),
+                    traffic_over_algorithmic=(traffic / w.bytes) if traffic else None,
+                    modeled_bytes=modeled,
                     per_launch_units=f"{F} token-expert rows x (d={cfg.d}, m={cfg.m})")
 
     extras = measure_extras(cfg, L, W2, dm, flush, pk, iters=args.extras_iters)
+    if cfg.name != "deepseek_v3" and not args.no_deepseek:
+        # the DeepSeek-V3-shaped layer (d = 7168, 256 routed experts + 1 shared, 22.6 GB of
+        # expert weights), both modes
+        extras["deepseek_v3"] = measure_layer_modes(synth.CONFIGS["deepseek_v3"], flush, pk,
+                                                    iters=min(args.extras_iters, 20))
 
     # ---- end to end through the public API with host buffers.  Every step copies its input
     # from pinned host memory and both layer outputs and the recorded route back; the copies of

@@ -23,7 +23,10 @@
  *    error before anything is launched.  Data-dependent problems found on the device (a replay
  *    index outside [0, N) or repeated within a token; a bounded device wait that ran out) are
  *    OR-ed into the caller's device status word as PR2_STATUS_* bits; the offending slot then
- *    contributes nothing.  With PR2_F_SYNC_STATUS in dims->flags the call synchronises the
+ *    contributes nothing.  After a timeout the layer output is unspecified: the kernels of
+ *    pr2_moe_forward that find PR2_STATUS_TIMEOUT in the word when they start (the grouped
+ *    GEMMs and the combine, which read tables an aborted dispatch may not have written) do no
+ *    work.  With PR2_F_SYNC_STATUS in dims->flags the call synchronises the
  *    stream, reads the status word and returns PR2_ERR_BAD_INDEX / PR2_ERR_TIMEOUT.  No C++
  *    exception crosses this ABI and no kernel traps.
  *  - Supported shapes: 1 <= k <= min(N, 32).  PR2_FP32 runs exact-fp32 SIMT kernels (N <= 256).

@@ -97,6 +97,17 @@ def expert_mlp_work(rows: int, d: int, m: int, experts_hit: int, dtype: str = "b
     return KernelWork(g.bytes + dn.bytes, g.flops + dn.flops)
 
 
+def expert_mlp_algorithmic_work(rows: int, d: int, m: int, experts_hit: int,
+                                dtype: str = "bf16", a_rows: int | None = None) -> KernelWork:
+    """Compulsory work of the grouped gated-MLP stage (gate/up + SwiGLU + down) as a fused
+    minimum: the weights of every expert hit (3*d*m each) and the distinct A rows (`a_rows`,
+    default `rows`) cross HBM once; the intermediates H [rows, m] and Y [rows, d] are not
+    counted (a fused layer keeps them on chip).  FLOPs 6*rows*d*m (App. E.2)."""
+    e = _esz(dtype)
+    a = rows if a_rows is None else a_rows
+    return KernelWork(a * d * e + experts_hit * 3 * d * m * e, 6 * rows * d * m)
+
+
 def combine_work(T: int, d: int, k: int, n_shared: int = 0, dtype: str = "bf16") -> KernelWork:
     """out[t] = sum_s g[t,s] Y[inv[t,s]] (+ shared rows): read Y, gates, inv; write out."""
     e = _esz(dtype)

@@ -470,9 +470,11 @@ template <typename T, int V, int KMAX>  // V elements per 16-byte vector, k <= K
 __global__ void __launch_bounds__(256)
     combine_kernel(const T* __restrict__ Y, const T* __restrict__ Ys,
                    const int32_t* __restrict__ inv, const float* __restrict__ gates, int64_t Tn,
-                   int k, int d, int n_shared, const T* residual, T* out) {
+                   int k, int d, int n_shared, const T* residual, T* out,
+                   const int32_t* status) {
   pdl_wait();
   pdl_trigger();
+  if (status_timed_out(status)) return;  // dispatch gave up: inv may be unwritten
   const int lane = threadIdx.x & 31;
   const int64_t warp0 = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
@@ -587,9 +589,11 @@ __global__ void __launch_bounds__(kCbThreads, 1)
     abort_flag_s = 0;
     fence_mbar_init();
   }
-  __syncthreads();
   pdl_wait();
   pdl_trigger();
+  if (threadIdx.x == 0) abort_flag_s = status_timed_out(status) ? 1 : 0;  // no tables to read
+  __syncthreads();
+  if (abort_flag_s) return;
   const int nvec = d / 8;
   if (warp == 0) {
     // ---------------- producer ----------------
@@ -761,6 +765,7 @@ cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st)
 
 cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st) {
   if (a.T == 0) return cudaSuccess;
+  const int32_t* status = a.status;
   int64_t blocks = (a.T + 7) / 8;
   const int64_t cap = static_cast<int64_t>(num_sms) * 8;
   if (blocks > cap) blocks = cap;
@@ -785,16 +790,16 @@ cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st) {
     }
     // (bf16 layers have k <= 8, checked at the ABI)
     return launch_pdl(combine_kernel<__nv_bfloat16, 8, 8>, grid, block, 0, st, 1, Y, Ys, a.inv,
-                      a.gates, a.T, a.k, a.d, a.n_shared, res, out);
+                      a.gates, a.T, a.k, a.d, a.n_shared, res, out, status);
   }
   auto* Y = static_cast<const float*>(a.Y);
   auto* Ys = static_cast<const float*>(a.Ys);
   auto* out = static_cast<float*>(a.out);
   auto* res = static_cast<const float*>(a.residual);
   return a.k <= 8 ? launch_pdl(combine_kernel<float, 4, 8>, grid, block, 0, st, 1, Y, Ys, a.inv,
-                               a.gates, a.T, a.k, a.d, a.n_shared, res, out)
+                               a.gates, a.T, a.k, a.d, a.n_shared, res, out, status)
                   : launch_pdl(combine_kernel<float, 4, 32>, grid, block, 0, st, 1, Y, Ys, a.inv,
-                               a.gates, a.T, a.k, a.d, a.n_shared, res, out);
+                               a.gates, a.T, a.k, a.d, a.n_shared, res, out, status);
 }
 
 }  // namespace pr2

@@ -16,10 +16,11 @@ __global__ void __launch_bounds__(kCols)
     expert_simt_kernel(int swiglu, const float* __restrict__ A, const float* __restrict__ W0,
                        const float* __restrict__ W1, const TileEntry* __restrict__ tiles,
                        const int32_t* __restrict__ num_tiles, int K, int n_out, int b_rows,
-                       float* __restrict__ out) {
+                       float* __restrict__ out, const int32_t* status) {
   pdl_wait();
   pdl_trigger();
-  if (static_cast<int>(blockIdx.x) >= *num_tiles) return;
+  // blockIdx.x < max_tiles by the grid; a dispatch that timed out leaves the table unwritten
+  if (status_timed_out(status) || static_cast<int>(blockIdx.x) >= *num_tiles) return;
   const TileEntry te = tiles[blockIdx.x];
   const int c = blockIdx.y * kCols + threadIdx.x;
   if (c >= n_out) return;
@@ -49,7 +50,8 @@ cudaError_t launch_expert_simt(bool swiglu, const float* A, const float* Wb0, co
   dim3 grid(g.max_tiles, (g.n_out + kCols - 1) / kCols);
   return launch_pdl(expert_simt_kernel, grid, dim3(kCols), 0, st, 1, swiglu ? 1 : 0, A, Wb0, Wb1,
                     static_cast<const TileEntry*>(g.tiles), g.num_tiles, g.K, g.n_out,
-                    g.b_rows_per_expert, static_cast<float*>(g.out));
+                    g.b_rows_per_expert, static_cast<float*>(g.out),
+                    static_cast<const int32_t*>(g.status));
 }
 
 }  // namespace pr2

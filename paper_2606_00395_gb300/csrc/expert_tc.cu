@@ -263,9 +263,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
   pdl_wait();  // the tile table and the A operand come from the previous kernels
   pdl_trigger();
+  __shared__ int nm_s;
+  if (threadIdx.x == 0) {
+    const int nm = status_timed_out(gs.status) ? 0 : *gs.num_tiles;
+    nm_s = nm < 0 ? 0 : (nm > gs.max_tiles ? gs.max_tiles : nm);
+  }
+  __syncthreads();
   Launch L;
   L.kind = kKind;
-  L.nm = *gs.num_tiles;
+  L.nm = nm_s;  // dispatch's count, never above the host bound; 0 after a timeout
   L.n1 = kHas0 ? (g0.n_out + kBN / 2 - 1) / (kBN / 2) : 0;
   L.n2 = kHas1 ? (g1.n_out + kBN - 1) / kBN : 0;
   L.num_jobs = L.nm * (L.n1 + L.n2);

@@ -181,6 +181,13 @@ __device__ __forceinline__ int ld_acquire_gpu(const int* p) {
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
+// Whether an earlier kernel of the call recorded PR2_STATUS_TIMEOUT in the status word (read
+// after pdl_wait).  The kernels that consume dispatch's tables (grouped GEMMs, combine) then do
+// nothing: a dispatch whose grid barrier gave up may have left those tables unwritten.
+__device__ __forceinline__ bool status_timed_out(const int32_t* status) {
+  if (status == nullptr) return false;
+  return (*reinterpret_cast<const volatile int32_t*>(status) & PR2_STATUS_TIMEOUT) != 0;
+}
 __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }

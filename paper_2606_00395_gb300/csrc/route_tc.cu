@@ -701,7 +701,7 @@ cudaError_t launch_any(int mode, const CUtensorMap& tm_h, const CUtensorMap& tm_
 }
 
 // CTAs of route_tc_kernel<mode, 1> with the compact layout that fit on one SM by its shared
-// memory, registers and threads (0 on error).  Counted from the kernel's attributes and the
+// memory, registers, threads and TMEM columns (0 on error).  Counted from the kernel's attributes and the
 // device limits: the occupancy query answers 1 for this kernel although two CTAs do run on
 // one SM side by side (a per-CTA %smid / %globaltimer record of a T = 32768 launch).
 template <int kMode>
@@ -726,6 +726,11 @@ int compact_blocks_per_sm(int N) {
   int n = static_cast<int>(static_cast<size_t>(smem_sm) / smem);
   if (regs > 0 && regs_sm / regs < n) n = regs_sm / regs;
   if (threads_sm / kThreads < n) n = threads_sm / kThreads;
+  // each CTA holds its accumulator columns for its whole life: more CTAs than fit in the SM's
+  // 512 TMEM columns would only wait in tcgen05.alloc for a neighbour to leave
+  const int b_rows = route_layout(N, kMode == kModePredict, true).b_rows;
+  const int by_tmem = static_cast<int>(512u / tmem_cols_for(b_rows));
+  if (by_tmem < n) n = by_tmem;
   return n;
 }
 

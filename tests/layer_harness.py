@@ -121,3 +121,40 @@ def compact_experts(L, idx_rows, tokens=None):
     Wd = cpu(L["W_down"].index_select(0, sel))
     new_idx = np.vectorize(lambda e: remap.get(int(e), -1))(np.asarray(idx_rows)).astype(np.int32)
     return Wg, Wu, Wd, new_idx
+
+
+def oracle_forward_rows(L, toks, idx_rows, gates_rows, with_shared=True,
+                        max_host_bytes=4 << 30):
+    """fp64 oracle layer output for the tokens ``toks`` of a (possibly very large) layer whose
+    tensors live on the GPU, with the routes ``idx_rows`` / gates ``gates_rows`` of those tokens.
+
+    Only the experts the rows reference are copied to the host, at most ``max_host_bytes`` of
+    expert weights at a time: when they do not fit at once (the DeepSeek-V3-shaped layer's 256
+    experts are 22.6 GB), the referenced experts are split into groups, the oracle runs once per
+    group with the other groups' slots marked invalid (the oracle skips them), and the group
+    outputs are added.  Each token's slots are thereby summed in group order instead of slot
+    order: a reassociation of at most k fp64 terms.  The shared experts enter with the first
+    group only."""
+    idx_rows = np.asarray(idx_rows)
+    used = sorted(set(int(e) for e in idx_rows.reshape(-1) if 0 <= e < L["W_gate"].shape[0]))
+    per_expert = 3 * L["W_gate"].shape[1] * L["W_gate"].shape[2] * L["W_gate"].element_size()
+    group = max(1, int(max_host_bytes // per_expert))
+    sel_t = torch.as_tensor(np.asarray(toks), dtype=torch.long, device=L["x"].device)
+    x_s = cpu(L["x"].index_select(0, sel_t))
+    sh = [cpu(L[n]) if (with_shared and L.get(n) is not None) else None
+          for n in ("Ws_gate", "Ws_up", "Ws_down")]
+    out = None
+    for g0 in range(0, max(len(used), 1), group):
+        chunk = used[g0:g0 + group]
+        remap = {e: i for i, e in enumerate(chunk)}
+        sel = torch.tensor(chunk if chunk else [0], dtype=torch.long, device=L["W_gate"].device)
+        Wg = cpu(L["W_gate"].index_select(0, sel))
+        Wu = cpu(L["W_up"].index_select(0, sel))
+        Wd = cpu(L["W_down"].index_select(0, sel))
+        idx_c = np.vectorize(lambda e: remap.get(int(e), -1))(idx_rows).astype(np.int32)
+        part = oracle.moe_forward(x_s, idx_c, gates_rows, Wg, Wu, Wd,
+                                  *(sh if g0 == 0 else (None, None, None)))
+        out = part if out is None else out + part
+        del Wg, Wu, Wd
+    return out
+

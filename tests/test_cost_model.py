@@ -37,6 +37,10 @@ def test_kernel_work_counts_each_tensor_once():
     assert g.bytes - gg.bytes == (32768 - 4096) * 2048 * 2 and gg.flops == g.flops
     mlp = cost.expert_mlp_work(32768, 2048, 768, 128, a_rows=4096)
     assert mlp.bytes == gg.bytes + dn.bytes and mlp.flops == g.flops + dn.flops
+    # the fused minimum of the expert stage: h once and the hit experts' weights, no H / Y
+    alg = cost.expert_mlp_algorithmic_work(32768, 2048, 768, 128, a_rows=4096)
+    assert alg.bytes == 4096 * 2048 * 2 + 128 * 3 * 2048 * 768 * 2 and alg.flops == mlp.flops
+    assert mlp.bytes - alg.bytes == 2 * 32768 * 768 * 2 + 32768 * 2048 * 2  # H out+in, Y out
     assert cost.dispatch_work(4096, 2048, 8).bytes == 3 * 4096 * 8 * 4
     assert (cost.dispatch_work(4096, 2048, 8, "fp32", gather=True).bytes
             == 3 * 4096 * 8 * 4 + 4096 * 2048 * 4 + 32768 * 2048 * 4)

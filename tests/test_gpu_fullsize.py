@@ -1,7 +1,14 @@
 """GPU parity at the full workload sizes (Qwen3-30B-A3B-shaped layer, its decode batch, the
-Zipf-skewed long replay and the DeepSeek-V3-shaped layer).  Inputs are drawn on the GPU;
-routes, counts and permutations are checked on every token, layer outputs on a seeded sample of
-tokens the oracle computes one by one."""
+Zipf-skewed long replay and the DeepSeek-V3-shaped layer).  Inputs are drawn on the GPU.
+
+* Qwen3-shaped layer (T = 4096): every route, gate, logit, replay gate, replay probability,
+  count, permutation and layer output of both modes against the oracle.
+* Decode batch (T = 256): everything, in full.
+* Long replay (T = 32768) and DeepSeek-V3-shaped layer (T = 8192): every count and permutation
+  (bit-exact), routes / gates / probabilities and layer outputs on a seeded sample of 512
+  tokens that the oracle computes one by one.
+Rollout outputs are compared with the oracle recomputed on the GPU's own route, weighted by the
+oracle's probabilities there, so near-tie tokens are compared too."""
 import numpy as np
 import pytest
 import torch
@@ -13,6 +20,8 @@ from tests import layer_harness as H
 
 pytestmark = pytest.mark.gpu
 
+SAMPLE = 512  # tokens compared one by one on the layers too large for a full oracle pass
+
 
 @pytest.fixture(scope="module", autouse=True)
 def _lib():
@@ -23,19 +32,8 @@ def _lib():
     B.load()
 
 
-def _sample_output_check(cfg, L, idx, gates, out, n_tok, seed=0):
-    toks = synth.make_token_sample(cfg.T, n_tok, seed).numpy()
-    idx_s = np.asarray(idx)[toks]
-    Wg, Wu, Wd, idx_c = H.compact_experts(L, idx_s)
-    x_s = H.cpu(L["x"][torch.from_numpy(toks).to(L["x"].device)])
-    sh = [H.cpu(L[n]) if L[n] is not None else None for n in ("Ws_gate", "Ws_up", "Ws_down")]
-    want = oracle.moe_forward(x_s, idx_c, np.asarray(gates)[toks], Wg, Wu, Wd, *sh)
-    got = H.cpu(out).float().numpy()[toks]
-    return H.normwise_close(got, want, H.OUT_TOL[cfg.dtype])
-
-
 def _routing_check(cfg, L, g, sample=None):
-    """Full (or sampled) route comparison; returns (exempt, checked) token counts."""
+    """Full (or sampled) route comparison; returns (exempt, checked, oracle result)."""
     x, idx, gates, logits = L["x"], H.cpu(g["idx"]).numpy(), H.cpu(g["gates"]).numpy(), \
         H.cpu(g["logits"]).numpy()
     if sample is not None:
@@ -49,35 +47,55 @@ def _routing_check(cfg, L, g, sample=None):
     return exempt, idx.shape[0], orc
 
 
-def test_qwen3_layer_both_modes():
+def _permutation_check(cfg, f, idx):
+    operm = oracle.permute(np.asarray(idx), cfg.N)
+    assert np.array_equal(H.cpu(f["counts"]).numpy(), operm["counts"])
+    nvalid = int(operm["offsets"][-1])
+    assert np.array_equal(H.cpu(f["perm"]).numpy()[:nvalid], operm["perm"])
+    return operm
+
+
+def _output_check(cfg, L, toks, idx_rows, gates_rows, out):
+    want = H.oracle_forward_rows(L, toks, idx_rows, gates_rows)
+    got = H.cpu(out).float().numpy()[np.asarray(toks)]
+    return H.normwise_close(got, want, H.OUT_TOL[cfg.dtype])
+
+
+def test_qwen3_layer_both_modes_in_full():
+    """The bench workload, every output of both modes: rollout on the GPU's own route, then
+    replay of the oracle's recorded route with the drifted router (Sec. 4.1)."""
     cfg = synth.CONFIGS["qwen3_30b_a3b"]
     L = synth.make_layer(cfg, device="cuda")
+    everyone = np.arange(cfg.T)
+    # ---- rollout (Eqs. pr2_predict, pr2_route, pr2_old_output)
     g = H.gpu_predict(cfg, L)
     exempt, n, orc = _routing_check(cfg, L, g)
-    print(f"qwen3 rollout: {exempt}/{n} near-tie tokens")
-    # replay the oracle's recorded route with the drifted router; permutation bit-exact
+    gidx = H.cpu(g["idx"]).numpy()
+    f_roll = H.gpu_forward(cfg, L, g["idx"], g["gates"])
+    assert f_roll["code"] == 0 and int(f_roll["status"].item()) == 0
+    _permutation_check(cfg, f_roll, gidx)
+    err_roll = _output_check(cfg, L, everyone, gidx,
+                             np.take_along_axis(orc["probs"], gidx, 1), f_roll["out"])
+    # ---- replay (Eq. pr2_output): gates and probabilities of every token
     W2 = synth.make_drifted_router(L["W_router"])
     idx_rec = torch.from_numpy(orc["idx"]).cuda()
-    r = H.gpu_replay(cfg, L, W2, idx_rec, probs=False)
-    toks = synth.make_token_sample(cfg.T, 256, 1).numpy()
-    orep = oracle.route_replay(H.cpu(L["x"])[toks], H.cpu(W2), orc["idx"][toks])
-    H.rowwise_close(H.cpu(r["gates"]).numpy()[toks], orep["gates"])
-    f = H.gpu_forward(cfg, L, idx_rec, r["gates"])
-    assert f["code"] == 0 and int(f["status"].item()) == 0
-    operm = oracle.permute(orc["idx"], cfg.N)
-    assert np.array_equal(H.cpu(f["counts"]).numpy(), operm["counts"])
-    assert np.array_equal(H.cpu(f["perm"]).numpy(), operm["perm"])
-    err = _sample_output_check(cfg, L, orc["idx"], H.cpu(r["gates"]).numpy(), f["out"], 48)
-    # rollout output on the GPU's own route, sampled
-    f2 = H.gpu_forward(cfg, L, g["idx"], g["gates"])
-    err2 = _sample_output_check(cfg, L, H.cpu(g["idx"]).numpy(), H.cpu(g["gates"]).numpy(),
-                                f2["out"], 48, seed=4)
-    print(f"qwen3 output error replay {err:.2e} rollout {err2:.2e}")
+    r = H.gpu_replay(cfg, L, W2, idx_rec, probs=True)
+    assert int(r["status"].item()) == 0
+    orep = oracle.route_replay(H.cpu(L["x"]), H.cpu(W2), orc["idx"])
+    H.rowwise_close(H.cpu(r["gates"]).numpy(), orep["gates"])
+    H.rowwise_close(H.cpu(r["probs"]).numpy(), orep["probs"])
+    f_rep = H.gpu_forward(cfg, L, idx_rec, r["gates"])
+    assert f_rep["code"] == 0 and int(f_rep["status"].item()) == 0
+    _permutation_check(cfg, f_rep, orc["idx"])
+    err_rep = _output_check(cfg, L, everyone, orc["idx"], orep["gates"], f_rep["out"])
+    print(f"qwen3: {exempt}/{n} near ties; output error rollout {err_roll:.2e}, "
+          f"replay {err_rep:.2e} (all {cfg.T} tokens)")
 
 
 def test_qwen3_shape_ragged_batch():
     """The Qwen3-shaped layer with T = 4001 (the last token tile 33 rows): every route against
-    the oracle, counts and permutation bit-exact, layer outputs on a token sample."""
+    the oracle, counts and permutation bit-exact, layer outputs on a token sample that includes
+    the ragged tile's end."""
     cfg = synth.CONFIGS["qwen3_30b_a3b"].scaled(4001)
     L = synth.make_layer(cfg, device="cuda")
     g = H.gpu_predict(cfg, L)
@@ -85,16 +103,11 @@ def test_qwen3_shape_ragged_batch():
     f = H.gpu_forward(cfg, L, g["idx"], g["gates"])
     assert f["code"] == 0 and int(f["status"].item()) == 0
     gidx = H.cpu(g["idx"]).numpy()
-    operm = oracle.permute(gidx, cfg.N)
-    assert np.array_equal(H.cpu(f["counts"]).numpy(), operm["counts"])
-    assert np.array_equal(H.cpu(f["perm"]).numpy(), operm["perm"])
-    toks = np.unique(np.concatenate([synth.make_token_sample(cfg.T, 40, 7).numpy(),
-                                     np.arange(cfg.T - 8, cfg.T)]))  # + the ragged tile's end
-    idx_s = gidx[toks]
-    Wg, Wu, Wd, idx_c = H.compact_experts(L, idx_s)
-    want = oracle.moe_forward(H.cpu(L["x"])[toks], idx_c, H.cpu(g["gates"]).numpy()[toks],
-                              Wg, Wu, Wd)
-    err = H.normwise_close(H.cpu(f["out"]).float().numpy()[toks], want, H.OUT_TOL[cfg.dtype])
+    _permutation_check(cfg, f, gidx)
+    toks = np.unique(np.concatenate([synth.make_token_sample(cfg.T, 256, 7).numpy(),
+                                     np.arange(cfg.T - 40, cfg.T)]))
+    err = _output_check(cfg, L, toks, gidx[toks],
+                        np.take_along_axis(orc["probs"], gidx, 1)[toks], f["out"])
     print(f"qwen3 T=4001: {exempt}/{n} near ties, output error {err:.2e}")
 
 
@@ -104,12 +117,12 @@ def test_qwen3_decode_batch_rollout():
     g = H.gpu_predict(cfg, L)
     exempt, n, orc = _routing_check(cfg, L, g)
     f = H.gpu_forward(cfg, L, g["idx"], g["gates"])
-    assert f["code"] == 0
+    assert f["code"] == 0 and int(f["status"].item()) == 0
     gidx = H.cpu(g["idx"]).numpy()
-    operm = oracle.permute(gidx, cfg.N)
-    assert np.array_equal(H.cpu(f["perm"]).numpy(), operm["perm"])
-    err = _sample_output_check(cfg, L, gidx, H.cpu(g["gates"]).numpy(), f["out"], 64)
-    print(f"decode: {exempt}/{n} near ties, output error {err:.2e}")
+    _permutation_check(cfg, f, gidx)
+    err = _output_check(cfg, L, np.arange(cfg.T), gidx,
+                        np.take_along_axis(orc["probs"], gidx, 1), f["out"])
+    print(f"decode: {exempt}/{n} near ties, output error {err:.2e} (all tokens)")
 
 
 def test_long_replay_with_zipf_routes():
@@ -117,19 +130,20 @@ def test_long_replay_with_zipf_routes():
     L = synth.make_layer(cfg, device="cuda")
     idx = synth.make_zipf_routes(cfg.T, cfg.N, cfg.k, cfg.zipf_s)
     idx_d = idx.cuda()
-    r = H.gpu_replay(cfg, L, L["W_router"], idx_d, probs=False)
-    toks = synth.make_token_sample(cfg.T, 256, 2).numpy()
+    r = H.gpu_replay(cfg, L, L["W_router"], idx_d, probs=True)
+    assert int(r["status"].item()) == 0
+    toks = synth.make_token_sample(cfg.T, SAMPLE, 2).numpy()
     orep = oracle.route_replay(H.cpu(L["x"])[toks], H.cpu(L["W_router"]), idx.numpy()[toks])
     H.rowwise_close(H.cpu(r["gates"]).numpy()[toks], orep["gates"])
+    H.rowwise_close(H.cpu(r["probs"]).numpy()[toks], orep["probs"])
     f = H.gpu_forward(cfg, L, idx_d, r["gates"])
     assert f["code"] == 0 and int(f["status"].item()) == 0
-    operm = oracle.permute(idx.numpy(), cfg.N)
-    counts = H.cpu(f["counts"]).numpy()
-    assert np.array_equal(counts, operm["counts"])
-    assert np.array_equal(H.cpu(f["perm"]).numpy(), operm["perm"])
+    operm = _permutation_check(cfg, f, idx.numpy())
+    counts = operm["counts"]
     assert counts.max() > 50 * counts.min()  # the load really is skewed
-    err = _sample_output_check(cfg, L, idx.numpy(), H.cpu(r["gates"]).numpy(), f["out"], 24)
-    print(f"zipf counts {counts.min()}..{counts.max()}, output error {err:.2e}")
+    err = _output_check(cfg, L, toks, idx.numpy()[toks], orep["gates"], f["out"])
+    print(f"zipf counts {counts.min()}..{counts.max()}, output error {err:.2e} "
+          f"({len(toks)} tokens)")
 
 
 @pytest.mark.parametrize("T", [32768, 20001])
@@ -151,17 +165,34 @@ def test_long_batch_routing_both_modes(T):
     print(f"long batch routing: {exempt}/{n} near ties (sampled)")
 
 
-def test_deepseek_v3_layer_with_shared_expert():
+def test_deepseek_v3_layer_both_modes():
+    """The DeepSeek-V3-shaped layer (T = 8192, d = 7168, 256 routed experts + 1 shared, top-8,
+    m = 2048) in both modes: rollout on the GPU's own route, then replay of that route with the
+    drifted router (Sec. 4.1; the shared expert of App. E.2 added with weight 1).  Every count
+    and permutation bit-exact; routes, gates, probabilities and outputs on 512 tokens."""
     cfg = synth.CONFIGS["deepseek_v3"]
     L = synth.make_layer(cfg, device="cuda")
+    sample = synth.make_token_sample(cfg.T, SAMPLE, 5).numpy()
+    # ---- rollout
     g = H.gpu_predict(cfg, L)
-    sample = synth.make_token_sample(cfg.T, 512, 5).numpy()
-    exempt, n, _ = _routing_check(cfg, L, g, sample=sample)
-    f = H.gpu_forward(cfg, L, g["idx"], g["gates"])
-    assert f["code"] == 0 and int(f["status"].item()) == 0
+    exempt, n, orc = _routing_check(cfg, L, g, sample=sample)
     gidx = H.cpu(g["idx"]).numpy()
-    operm = oracle.permute(gidx, cfg.N)
-    assert np.array_equal(H.cpu(f["counts"]).numpy(), operm["counts"])
-    assert np.array_equal(H.cpu(f["perm"]).numpy(), operm["perm"])
-    err = _sample_output_check(cfg, L, gidx, H.cpu(g["gates"]).numpy(), f["out"], 6)
-    print(f"deepseek: {exempt}/{n} near ties (sampled), output error {err:.2e}")
+    f_roll = H.gpu_forward(cfg, L, g["idx"], g["gates"])
+    assert f_roll["code"] == 0 and int(f_roll["status"].item()) == 0
+    _permutation_check(cfg, f_roll, gidx)
+    err_roll = _output_check(cfg, L, sample, gidx[sample],
+                             np.take_along_axis(orc["probs"], gidx[sample], 1), f_roll["out"])
+    # ---- replay of the recorded route with the drifted router
+    W2 = synth.make_drifted_router(L["W_router"])
+    r = H.gpu_replay(cfg, L, W2, g["idx"], probs=True)
+    assert int(r["status"].item()) == 0
+    sel = torch.from_numpy(sample).cuda()
+    orep = oracle.route_replay(H.cpu(L["x"][sel]), H.cpu(W2), gidx[sample])
+    H.rowwise_close(H.cpu(r["gates"]).numpy()[sample], orep["gates"])
+    H.rowwise_close(H.cpu(r["probs"]).numpy()[sample], orep["probs"])
+    f_rep = H.gpu_forward(cfg, L, g["idx"], r["gates"])
+    assert f_rep["code"] == 0 and int(f_rep["status"].item()) == 0
+    _permutation_check(cfg, f_rep, gidx)
+    err_rep = _output_check(cfg, L, sample, gidx[sample], orep["gates"], f_rep["out"])
+    print(f"deepseek: {exempt}/{n} near ties (sampled); output error rollout {err_roll:.2e}, "
+          f"replay {err_rep:.2e} ({len(sample)} tokens)")
