@@ -428,7 +428,7 @@ pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* 
   DispatchArgs da{idx,       dm.T,       dm.k,      dm.N,    dm.d,   es,     dm.n_shared,
                   w.blk_hist, w.counts,  w.offsets, w.perm,  w.inv,  w.tiles, w.num_tiles,
                   w.stiles1, w.stiles2,  h,         w.xperm, status, w.sync_ctr,
-                  dm.dtype == PR2_BF16 ? w.ready : nullptr};
+                  dm.dtype == PR2_BF16 ? w.ready : nullptr, kTileM};
   // (w.xperm is nullptr on the bf16 path: dispatch then launches no gather)
   if (err == cudaSuccess) err = launch_dispatch(da, num_sms, st);
   mark(events ? events->dispatched : nullptr);

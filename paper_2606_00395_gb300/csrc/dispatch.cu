@@ -93,13 +93,15 @@ __device__ __forceinline__ int block_exclusive_scan(int v, int* sh, int* total) 
   return incl - v;
 }
 
-// The grouped GEMM's M-tile table (entry i belongs to the expert whose tile range contains i;
-// its per-M-tile readiness counter is cleared) and the static tile tables of the shared experts
+// The grouped GEMM's tile table: each expert's rows split into ceil(rows / tile_rows) tiles of
+// near-equal size (entry i belongs to the expert whose tile range contains i; its per-tile
+// readiness counter is cleared) and the static tile tables of the shared experts
 // (every token: gate/up reads rows of h, down rows of Hs), from the experts' row offsets ex_off
 // and first tiles ex_tile (N + 1 entries each, in shared memory); num_tiles[0..1] = their
 // lengths.  Called by every thread of one block.
-__device__ void write_tile_tables(int N, int64_t T, int n_shared, const int* ex_off,
-                                  const int* ex_tile, TileEntry* __restrict__ tiles,
+__device__ void write_tile_tables(int N, int64_t T, int n_shared, int tile_rows,
+                                  const int* ex_off, const int* ex_tile,
+                                  TileEntry* __restrict__ tiles,
                                   int32_t* __restrict__ num_tiles,
                                   TileEntry* __restrict__ stiles1,
                                   TileEntry* __restrict__ stiles2, int32_t* __restrict__ ready) {
@@ -116,10 +118,14 @@ __device__ void write_tile_tables(int N, int64_t T, int n_shared, const int* ex_
       const int mid = (lo + hi + 1) >> 1;
       if (ex_tile[mid] <= i) lo = mid; else hi = mid - 1;
     }
+    // the expert's c rows split into nch = ceil(c / tile_rows) tiles of near-equal size
     const int j = i - ex_tile[lo];
-    const int r0 = ex_off[lo] + j * kTileM;
+    const int nch = ex_tile[lo + 1] - ex_tile[lo];
+    const int c = ex_off[lo + 1] - ex_off[lo];
+    const int sz = (c + nch - 1) / nch;
+    const int r0 = ex_off[lo] + j * sz;
     const int left = ex_off[lo + 1] - r0;
-    tiles[i] = TileEntry{lo, r0, left < kTileM ? left : kTileM, r0};
+    tiles[i] = TileEntry{lo, r0, left < sz ? left : sz, r0};
     if (ready != nullptr) ready[i] = 0;  // per M-tile counter of the fused expert GEMM
   }
   for (int i = tid; i < n_shared * mt_T; i += blockDim.x) {
@@ -136,6 +142,7 @@ __device__ void write_tile_tables(int N, int64_t T, int n_shared, const int* ex_
 // block range of group g, so the per-expert scans over blocks run G-way parallel.
 __global__ void __launch_bounds__(1024)
     scan_kernel(int32_t* __restrict__ blk_hist, int nblk, int N, int64_t T, int n_shared,
+                int tile_rows,
                 int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
                 TileEntry* __restrict__ tiles, int32_t* __restrict__ num_tiles,
                 TileEntry* __restrict__ stiles1, TileEntry* __restrict__ stiles2,
@@ -180,7 +187,7 @@ __global__ void __launch_bounds__(1024)
   __syncthreads();
   int all_rows, all_tiles;
   const int off = block_exclusive_scan(tid < N ? total : 0, sh, &all_rows);
-  const int ntile_e = tid < N ? (total + kTileM - 1) / kTileM : 0;
+  const int ntile_e = tid < N ? (total + tile_rows - 1) / tile_rows : 0;
   const int tstart = block_exclusive_scan(ntile_e, sh, &all_tiles);
   if (tid < N) {
     offsets[tid] = off;
@@ -208,7 +215,8 @@ __global__ void __launch_bounds__(1024)
       }
     }
   }
-  write_tile_tables(N, T, n_shared, ex_off, ex_tile, tiles, num_tiles, stiles1, stiles2, ready);
+  write_tile_tables(N, T, n_shared, tile_rows, ex_off, ex_tile, tiles, num_tiles, stiles1,
+                    stiles2, ready);
 }
 
 __global__ void __launch_bounds__(kDispatchChunk)
@@ -278,7 +286,7 @@ __device__ __forceinline__ int block256_exclusive_scan(int v, int* sh, int* tota
 // Hist, scan and place in one cooperative launch (N % 4 == 0, N <= 256; grid resident).
 __global__ void __launch_bounds__(kDispatchChunk)
     dispatch_fused_kernel(const int32_t* __restrict__ idx, int64_t F, int k, int N, int64_t T,
-                          int n_shared, int32_t* blk_hist, int32_t* __restrict__ counts,
+                          int n_shared, int tile_rows, int32_t* blk_hist, int32_t* __restrict__ counts,
                           int32_t* __restrict__ offsets, int32_t* __restrict__ perm,
                           int32_t* __restrict__ inv, TileEntry* __restrict__ tiles,
                           int32_t* __restrict__ num_tiles, TileEntry* __restrict__ stiles1,
@@ -376,7 +384,8 @@ __global__ void __launch_bounds__(kDispatchChunk)
   const int total = tid < N ? tot[tid] : 0;
   const int off = block256_exclusive_scan(total, sh, &all_rows);
   const int tstart =
-      block256_exclusive_scan(tid < N ? (total + kTileM - 1) / kTileM : 0, sh, &all_tiles);
+      block256_exclusive_scan(tid < N ? (total + tile_rows - 1) / tile_rows : 0, sh,
+                              &all_tiles);
   if (tid < N) {
     ex_off[tid] = off;
     ex_tile[tid] = tstart;
@@ -392,8 +401,8 @@ __global__ void __launch_bounds__(kDispatchChunk)
       offsets[tid] = off;
     }
     if (tid == 0) offsets[N] = all_rows;
-    write_tile_tables(N, T, n_shared, ex_off, ex_tile, tiles, num_tiles, stiles1, stiles2,
-                      ready);
+    write_tile_tables(N, T, n_shared, tile_rows, ex_off, ex_tile, tiles, num_tiles, stiles1,
+                      stiles2, ready);
   }
   // ---- 3. stable placement: per-warp bases, then ranks within the warp
   for (int x = tid; x < N; x += blockDim.x) {
@@ -729,7 +738,7 @@ cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st)
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     err = cudaLaunchKernelEx(&cfg, dispatch_fused_kernel, a.idx, F, a.k, a.N, a.T, a.n_shared,
-                             a.blk_hist, a.counts, a.offsets, a.perm, a.inv, a.tiles,
+                             a.tile_rows, a.blk_hist, a.counts, a.offsets, a.perm, a.inv, a.tiles,
                              a.num_tiles, a.stiles1, a.stiles2, a.sync_ctr, a.status, a.ready);
     if (err != cudaSuccess) return err;
   } else {
@@ -739,7 +748,7 @@ cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st)
       if (err != cudaSuccess) return err;
     }
     err = launch_pdl(scan_kernel, dim3(1), dim3(1024), 0, st, 1, a.blk_hist, nblk, a.N, a.T,
-                     a.n_shared, a.counts, a.offsets, a.tiles, a.num_tiles, a.stiles1,
+                     a.n_shared, a.tile_rows, a.counts, a.offsets, a.tiles, a.num_tiles, a.stiles1,
                      a.stiles2, a.ready);
     if (err != cudaSuccess) return err;
     if (nblk > 0) {

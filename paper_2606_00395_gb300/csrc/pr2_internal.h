@@ -113,6 +113,7 @@ struct DispatchArgs {
   unsigned int* sync_ctr;  // grid-barrier counter of the fused dispatch (zeroed per call)
   int32_t* ready;          // [max_mtiles] per M-tile counters of the fused GEMM, cleared here
                            // (nullable)
+  int tile_rows;           // most rows of one routed tile (an expert's rows are split evenly)
 };
 cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st);
 
