@@ -348,9 +348,9 @@ def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
         B.check(B.pr2_moe_forward(dm, L["x"], idx, gates, L["W_gate"], L["W_up"], L["W_down"],
                                   *sh, o1, workspace=wsl), "pr2_moe_forward")
         for Wr in (L["W_router"], W2):
-            B.check(B.pr2_route_replay(dm, L["x"], Wr, idx, rg, None), "pr2_route_replay")
-            B.check(B.pr2_moe_forward(dm, L["x"], idx, rg, L["W_gate"], L["W_up"], L["W_down"],
-                                      *sh, o1, workspace=wsl), "pr2_moe_forward")
+            B.check(B.pr2_moe_replay_forward(dm, L["x"], Wr, idx, rg, None, L["W_gate"],
+                                             L["W_up"], L["W_down"], *sh, o1, workspace=wsl),
+                    "pr2_moe_replay_forward")
     ms = timed(pr3)
     out["pr3_step"] = dict(ms=ms, tokens_per_s=cfg.T / (ms * 1e-3), passes=3, T=cfg.T)
     del wsl
@@ -445,12 +445,16 @@ def measure_layer_modes(cfg, flush, pk, iters, seed=0):
                                   *sh, o1, counts=counts, workspace=ws, status=status,
                                   events=st1), "pr2_moe_forward")
         marks[1].record()
-        B.check(B.pr2_route_replay(dm, L["x"], W2, idx, rg, None, status), "pr2_route_replay")
-        if len(marks) > 3:
+        if len(marks) > 3:  # per-kernel pass: routing and forward as separate calls
+            B.check(B.pr2_route_replay(dm, L["x"], W2, idx, rg, None, status), "pr2_route_replay")
             marks[4].record()
-        B.check(B.pr2_moe_forward(dm, L["x"], idx, rg, L["W_gate"], L["W_up"], L["W_down"],
-                                  *sh, o2, workspace=ws, status=status, events=st2),
-                "pr2_moe_forward")
+            B.check(B.pr2_moe_forward(dm, L["x"], idx, rg, L["W_gate"], L["W_up"], L["W_down"],
+                                      *sh, o2, workspace=ws, status=status, events=st2),
+                    "pr2_moe_forward")
+        else:  # the training-mode layer as one call
+            B.check(B.pr2_moe_replay_forward(dm, L["x"], W2, idx, rg, None, L["W_gate"],
+                                             L["W_up"], L["W_down"], *sh, o2, workspace=ws,
+                                             status=status), "pr2_moe_replay_forward")
         marks[2].record()
 
     sets = []
@@ -550,11 +554,20 @@ def run_pr2(args, rank, world, local_rank):
                                   L["Ws_gate"], L["Ws_up"], L["Ws_down"], out1, workspace=ws,
                                   status=status, events=evs[2]), "pr2_moe_forward")
         rec(evs[3])
-        B.check(B.pr2_route_replay(dm, x, W2, idx, rgates, None, status), "pr2_route_replay")
-        rec(evs[4])
-        B.check(B.pr2_moe_forward(dm, x, idx, rgates, L["W_gate"], L["W_up"], L["W_down"],
-                                  L["Ws_gate"], L["Ws_up"], L["Ws_down"], out2, workspace=ws,
-                                  status=status, events=evs[5]), "pr2_moe_forward")
+        if evs[4] is None:
+            # headline steps: the training-mode layer as one call (replay routing launched
+            # behind the expert GEMMs, same results as the two calls below)
+            B.check(B.pr2_moe_replay_forward(dm, x, W2, idx, rgates, None, L["W_gate"],
+                                             L["W_up"], L["W_down"], L["Ws_gate"], L["Ws_up"],
+                                             L["Ws_down"], out2, workspace=ws, status=status),
+                    "pr2_moe_replay_forward")
+        else:
+            # per-kernel breakdown pass: routing and forward as separate calls
+            B.check(B.pr2_route_replay(dm, x, W2, idx, rgates, None, status), "pr2_route_replay")
+            rec(evs[4])
+            B.check(B.pr2_moe_forward(dm, x, idx, rgates, L["W_gate"], L["W_up"], L["W_down"],
+                                      L["Ws_gate"], L["Ws_up"], L["Ws_down"], out2, workspace=ws,
+                                      status=status, events=evs[5]), "pr2_moe_forward")
         rec(evs[6])
 
     def make_evs(stages):
@@ -712,10 +725,10 @@ def run_pr2(args, rank, world, local_rank):
         B.check(B.pr2_moe_forward(dm, x, ixd[b], gates, L["W_gate"], L["W_up"], L["W_down"],
                                   L["Ws_gate"], L["Ws_up"], L["Ws_down"], o1[b], workspace=ws,
                                   status=status), "pr2_moe_forward")
-        B.check(B.pr2_route_replay(dm, x, W2, ixd[b], rgates, None, status), "pr2_route_replay")
-        B.check(B.pr2_moe_forward(dm, x, ixd[b], rgates, L["W_gate"], L["W_up"], L["W_down"],
-                                  L["Ws_gate"], L["Ws_up"], L["Ws_down"], o2[b], workspace=ws,
-                                  status=status), "pr2_moe_forward")
+        B.check(B.pr2_moe_replay_forward(dm, x, W2, ixd[b], rgates, None, L["W_gate"], L["W_up"],
+                                         L["W_down"], L["Ws_gate"], L["Ws_up"], L["Ws_down"],
+                                         o2[b], workspace=ws, status=status),
+                "pr2_moe_replay_forward")
 
     def d2h(b, comp_ev):
         with torch.cuda.stream(cs):

@@ -150,6 +150,23 @@ pr2_status pr2_moe_forward(const pr2_dims* dims, const void* h, const int32_t* i
                            const pr2_stage_events* events, void* stream);
 
 /*
+ * Training-mode layer in one call: pr2_route_replay followed by pr2_moe_forward on its gates
+ * (Sec. 4.1 "Replay During Training", Eq. pr2_output), with identical results.  Only the
+ * gate-weighted combine reads the replay gates, so the call launches dispatch and the expert
+ * GEMMs first and the replay routing behind them; on the tensor-core path the routing kernel
+ * runs on the SMs the GEMM's last CTAs free instead of in front of the whole layer.
+ * Arguments as in pr2_route_replay (W_router, idx, gates written, probs nullable) and
+ * pr2_moe_forward (the rest).  status_dev collects the bits of both steps.
+ */
+pr2_status pr2_moe_replay_forward(const pr2_dims* dims, const void* h, const void* W_router,
+                                  const int32_t* idx, float* gates, float* probs,
+                                  const void* W_gate, const void* W_up, const void* W_down,
+                                  const void* Ws_gate, const void* Ws_up, const void* Ws_down,
+                                  void* out, int32_t* counts, int32_t* perm, void* workspace,
+                                  size_t ws_bytes, int32_t* status_dev,
+                                  const pr2_stage_events* events, void* stream);
+
+/*
  * pr2_moe_forward without a caller-provided workspace.  The paper has no counterpart: this
  * entry point exists for callers that cannot allocate device memory where they run the layer
  * (a runtime whose pool owns all device memory, a hot path on which cudaMalloc/cudaFree and

@@ -145,7 +145,8 @@ pr2_status finish(cudaError_t err, uint32_t flags, int32_t* status_dev, cudaStre
 
 pr2_status route_common(const pr2_dims* dims, bool predict, const void* h, const void* W,
                         const void* Wp, const int32_t* idx_in, int32_t* idx_out, float* gates,
-                        float* aux, int64_t* near_tie, int32_t* status_dev, void* stream) {
+                        float* aux, int64_t* near_tie, int32_t* status_dev, void* stream,
+                        bool late_wait = false) {
   pr2_status s = check_dims(dims);
   if (s != PR2_OK) return s;
   const pr2_dims& dm = *dims;
@@ -192,6 +193,7 @@ pr2_status route_common(const pr2_dims* dims, bool predict, const void* h, const
     a.status = status_dev;
     a.norm = (dm.flags & PR2_F_NORMALIZE_TOPK) ? 1 : 0;
     a.compact = compact ? 1 : 0;
+    a.late_wait = late_wait ? 1 : 0;
     err = launch_route_tc(mode, tm_h, tm_w, tm_wp, a, split, st);
   }
   return finish(err, dm.flags, status_dev, st);
@@ -381,15 +383,24 @@ size_t pr2_moe_workspace_bytes(const pr2_dims* dims) {
 namespace pr2 {
 namespace {
 
+// Replay routing run inside the layer forward (pr2_moe_replay_forward): the current router and
+// the gates / probabilities it writes.
+struct ReplayRoute {
+  const void* W_router;
+  float* probs;
+};
+
 // The layer forward of pr2_moe_forward; `residual` (nullable, [T, d] in the layer dtype, may
-// alias `out`) is added to the combined output.
+// alias `out`) is added to the combined output.  With `replay`, the replay gates of the route
+// `idx` are computed into `gates` after the expert GEMMs and before the combine, which is the
+// only step that reads them.
 pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* idx,
                             const float* gates, const void* W_gate, const void* W_up,
                             const void* W_down, const void* Ws_gate, const void* Ws_up,
                             const void* Ws_down, void* out, const void* residual,
                             int32_t* counts, int32_t* perm, void* workspace, size_t ws_bytes,
                             int32_t* status_dev, const pr2_stage_events* events,
-                            void* stream) {
+                            void* stream, const ReplayRoute* replay = nullptr) {
   pr2_status s = check_dims(dims);
   if (s != PR2_OK) return s;
   const pr2_dims& dm = *dims;
@@ -488,6 +499,17 @@ pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* 
     mark(events ? events->down_done : nullptr);
   }
   if (err != cudaSuccess) return PR2_ERR_CUDA;
+  if (replay != nullptr) {
+    // Its inputs (h, the router, the route) are complete before the GEMMs start, so on the
+    // tensor-core path its CTAs take the SMs the GEMM's last CTAs free and wait for the GEMMs
+    // only before exiting; the combine launched behind it then sees both.
+    pr2_dims dr = dm;
+    dr.flags &= ~PR2_F_SYNC_STATUS;
+    s = route_common(&dr, false, h, replay->W_router, nullptr, idx, nullptr,
+                     const_cast<float*>(gates), replay->probs, nullptr, status, stream,
+                     dm.dtype == PR2_BF16);
+    if (s != PR2_OK) return s;
+  }
 
   CombineArgs ca{w.ybuf, dm.n_shared > 0 ? w.ys : nullptr, w.inv, gates, dm.T, dm.k, dm.d,
                  dm.n_shared, dm.dtype == PR2_BF16 ? 1 : 0, out, residual, status};
@@ -514,6 +536,26 @@ pr2_status pr2_moe_forward(const pr2_dims* dims, const void* h, const int32_t* i
   return moe_forward_impl(dims, h, idx, gates, W_gate, W_up, W_down, Ws_gate, Ws_up, Ws_down,
                           out, nullptr, counts, perm, workspace, ws_bytes, status_dev, events,
                           stream);
+}
+
+pr2_status pr2_moe_replay_forward(const pr2_dims* dims, const void* h, const void* W_router,
+                                  const int32_t* idx, float* gates, float* probs,
+                                  const void* W_gate, const void* W_up, const void* W_down,
+                                  const void* Ws_gate, const void* Ws_up, const void* Ws_down,
+                                  void* out, int32_t* counts, int32_t* perm, void* workspace,
+                                  size_t ws_bytes, int32_t* status_dev,
+                                  const pr2_stage_events* events, void* stream) {
+  pr2_status s = check_dims(dims);
+  if (s != PR2_OK) return s;
+  if (dims->T == 0) return PR2_OK;
+  // everything the routing step needs is checked here, before the forward launches anything
+  if (W_router == nullptr || gates == nullptr || !aligned16(W_router) ||
+      (probs != nullptr && !aligned16(probs)))
+    return PR2_ERR_INVALID_ARG;
+  const ReplayRoute rr{W_router, probs};
+  return moe_forward_impl(dims, h, idx, gates, W_gate, W_up, W_down, Ws_gate, Ws_up, Ws_down,
+                          out, nullptr, counts, perm, workspace, ws_bytes, status_dev, events,
+                          stream, &rr);
 }
 
 pr2_status pr2_rollout_layers(const pr2_dims* dims, int32_t L, void* h, const void* W_router,

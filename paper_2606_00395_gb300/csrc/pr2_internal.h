@@ -73,6 +73,8 @@ struct RouteTcArgs {
   int32_t* status;
   int norm;                // PR2_F_NORMALIZE_TOPK: gates divided by their sum over the route
   int compact;             // 1: half the pipeline stages, so two CTAs share an SM (split 1)
+  int late_wait;           // 1: the inputs are known ready; wait for the previous kernel only
+                           // before exiting (the launch overlaps it; see pr2_moe_replay_forward)
   // kModeLoss only (h = h_old, W = W_p)
   const float* p_old;      // [T, N] cached router logits
   const float* rho;        // [T_rho, N] teacher probabilities

@@ -219,7 +219,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  pdl_wait();  // h, the weights and the cached route may come from the previous kernels
+  // h, the weights and the cached route may come from the previous kernels.  With late_wait
+  // the caller guarantees they are complete already (the kernel before is a grouped GEMM whose
+  // own inputs came after them), so the CTAs start on the SMs that GEMM frees and wait for it
+  // only before they exit: a kernel launched after this one then sees the GEMM's results too.
+  if (!a.late_wait) pdl_wait();
   pdl_trigger();
 
   if (warp == 0) {
@@ -634,6 +638,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, ncols);
   }
+  if (a.late_wait) pdl_wait();
 }
 
 template <int kMode, int kSplit>

@@ -273,3 +273,42 @@ def test_all_invalid_route_gives_the_shared_experts_alone(n_shared):
         assert np.all(got == 0.0)
     else:
         H.normwise_close(got, want, H.OUT_TOL["bf16"])
+
+
+@pytest.mark.parametrize("name", ["tiny_fp32", "bf16_multitile", "bf16_partial_n",
+                                  "bf16_shared_n256", "bf16_one_token"])
+def test_replay_layer_call_equals_the_two_calls(name):
+    """pr2_moe_replay_forward (replay routing launched behind the expert GEMMs) writes exactly
+    what pr2_route_replay followed by pr2_moe_forward writes: gates, probabilities, counts,
+    permutation and layer output, bit for bit; an invalid cached slot is flagged the same way."""
+    cfg = SMALL[name]
+    L = synth.make_layer(cfg, seed=11)
+    Ld = H.to_dev(L)
+    W2 = synth.make_drifted_router(L["W_router"], seed=11).cuda()
+    g = H.gpu_predict(cfg, Ld)
+    idx = g["idx"].clone()
+    if cfg.T > 3:
+        idx[3, 0] = cfg.N  # one invalid slot
+    r = H.gpu_replay(cfg, Ld, W2, idx)
+    ref = H.gpu_forward(cfg, Ld, idx, r["gates"])
+    assert ref["code"] == 0
+    dm = H.dims_of(cfg)
+    gates = torch.full_like(r["gates"], float("nan"))
+    probs = torch.full_like(r["probs"], float("nan"))
+    out = torch.full_like(ref["out"], float("nan"))
+    counts = torch.full_like(ref["counts"], -1)
+    perm = torch.full_like(ref["perm"], -1)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    code = B.pr2_moe_replay_forward(dm, Ld["x"], W2, idx, gates, probs, Ld["W_gate"], Ld["W_up"],
+                                    Ld["W_down"], Ld["Ws_gate"], Ld["Ws_up"], Ld["Ws_down"], out,
+                                    counts=counts, perm=perm, workspace=B.alloc_workspace(dm),
+                                    status=status)
+    assert code == 0, B.pr2_strerror(code)
+    torch.cuda.synchronize()
+    assert torch.equal(gates, r["gates"]) and torch.equal(probs, r["probs"])
+    n_valid = int(ref["counts"].sum().item())  # perm entries past sum(counts) are unspecified
+    assert torch.equal(counts, ref["counts"]) and torch.equal(perm[:n_valid], ref["perm"][:n_valid])
+    assert torch.equal(out, ref["out"])
+    want_status = int(r["status"].item()) | int(ref["status"].item())
+    assert int(status.item()) == want_status
+    assert (want_status & B.PR2_STATUS_BAD_INDEX) == (B.PR2_STATUS_BAD_INDEX if cfg.T > 3 else 0)
