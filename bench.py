@@ -324,10 +324,11 @@ def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
                 "pr2_route_predict")
 
     def layer_d():
-        route_d()
-        B.check(B.pr2_moe_forward(ddm, xd, di, dgt, L["W_gate"], L["W_up"], L["W_down"],
-                                  L["Ws_gate"], L["Ws_up"], L["Ws_down"], do, workspace=dws,
-                                  status=status), "pr2_moe_forward")
+        B.check(B.pr2_moe_rollout_forward(ddm, xd, L["W_router"], L["W_pred"], di, dgt, dlg,
+                                          None, L["W_gate"], L["W_up"], L["W_down"],
+                                          L["Ws_gate"], L["Ws_up"], L["Ws_down"], do,
+                                          workspace=dws, status=status),
+                "pr2_moe_rollout_forward")
     ms = timed(route_d)
     report("decode_route_predict", ms, per_layer[0], T=Td, latency_us=ms * 1e3)
     ms = timed(layer_d)
@@ -342,11 +343,10 @@ def measure_extras(cfg, L, W2, dm, flush, pk, iters=50):
     wsl = B.alloc_workspace(dm)
 
     def pr3():
-        B.check(B.pr2_route_predict(dm, L["x"], L["W_router"], L["W_pred"], idx, gates, logits),
-                "pr2_route_predict")
         sh = (L["Ws_gate"], L["Ws_up"], L["Ws_down"])
-        B.check(B.pr2_moe_forward(dm, L["x"], idx, gates, L["W_gate"], L["W_up"], L["W_down"],
-                                  *sh, o1, workspace=wsl), "pr2_moe_forward")
+        B.check(B.pr2_moe_rollout_forward(dm, L["x"], L["W_router"], L["W_pred"], idx, gates,
+                                          logits, None, L["W_gate"], L["W_up"], L["W_down"],
+                                          *sh, o1, workspace=wsl), "pr2_moe_rollout_forward")
         for Wr in (L["W_router"], W2):
             B.check(B.pr2_moe_replay_forward(dm, L["x"], Wr, idx, rg, None, L["W_gate"],
                                              L["W_up"], L["W_down"], *sh, o1, workspace=wsl),
@@ -437,13 +437,19 @@ def measure_layer_modes(cfg, flush, pk, iters, seed=0):
 
     def one(marks, st1=None, st2=None):
         marks[0].record()
-        B.check(B.pr2_route_predict(dm, L["x"], L["W_router"], L["W_pred"], idx, gates, logits,
-                                    None, status), "pr2_route_predict")
-        if len(marks) > 3:
+        if len(marks) > 3:  # per-kernel pass: routing and forward as separate calls
+            B.check(B.pr2_route_predict(dm, L["x"], L["W_router"], L["W_pred"], idx, gates,
+                                        logits, None, status), "pr2_route_predict")
             marks[3].record()
-        B.check(B.pr2_moe_forward(dm, L["x"], idx, gates, L["W_gate"], L["W_up"], L["W_down"],
-                                  *sh, o1, counts=counts, workspace=ws, status=status,
-                                  events=st1), "pr2_moe_forward")
+            B.check(B.pr2_moe_forward(dm, L["x"], idx, gates, L["W_gate"], L["W_up"],
+                                      L["W_down"], *sh, o1, counts=counts, workspace=ws,
+                                      status=status, events=st1), "pr2_moe_forward")
+        else:  # the rollout-mode layer as one call
+            B.check(B.pr2_moe_rollout_forward(dm, L["x"], L["W_router"], L["W_pred"], idx,
+                                              gates, logits, None, L["W_gate"], L["W_up"],
+                                              L["W_down"], *sh, o1, counts=counts,
+                                              workspace=ws, status=status),
+                    "pr2_moe_rollout_forward")
         marks[1].record()
         if len(marks) > 3:  # per-kernel pass: routing and forward as separate calls
             B.check(B.pr2_route_replay(dm, L["x"], W2, idx, rg, None, status), "pr2_route_replay")
@@ -547,12 +553,23 @@ def run_pr2(args, rank, world, local_rank):
 
     def step(x, evs):
         rec(evs[0])
-        B.check(B.pr2_route_predict(dm, x, L["W_router"], L["W_pred"], idx, gates, logits, near,
-                                    status), "pr2_route_predict")
-        rec(evs[1])
-        B.check(B.pr2_moe_forward(dm, x, idx, gates, L["W_gate"], L["W_up"], L["W_down"],
-                                  L["Ws_gate"], L["Ws_up"], L["Ws_down"], out1, workspace=ws,
-                                  status=status, events=evs[2]), "pr2_moe_forward")
+        if evs[1] is None:
+            # headline steps: the rollout-mode layer as one call (dispatch from the routing
+            # kernel's histograms, same results as the two calls below)
+            B.check(B.pr2_moe_rollout_forward(dm, x, L["W_router"], L["W_pred"], idx, gates,
+                                              logits, near, L["W_gate"], L["W_up"], L["W_down"],
+                                              L["Ws_gate"], L["Ws_up"], L["Ws_down"], out1,
+                                              workspace=ws, status=status),
+                    "pr2_moe_rollout_forward")
+        else:
+            # per-kernel breakdown pass: routing and forward as separate calls
+            B.check(B.pr2_route_predict(dm, x, L["W_router"], L["W_pred"], idx, gates, logits,
+                                        near, status), "pr2_route_predict")
+            rec(evs[1])
+            B.check(B.pr2_moe_forward(dm, x, idx, gates, L["W_gate"], L["W_up"], L["W_down"],
+                                      L["Ws_gate"], L["Ws_up"], L["Ws_down"], out1,
+                                      workspace=ws, status=status, events=evs[2]),
+                    "pr2_moe_forward")
         rec(evs[3])
         if evs[4] is None:
             # headline steps: the training-mode layer as one call (replay routing launched
@@ -720,11 +737,11 @@ def run_pr2(args, rank, world, local_rank):
 
     def e2e_compute(b):
         x = xd[b]
-        B.check(B.pr2_route_predict(dm, x, L["W_router"], L["W_pred"], ixd[b], gates, logits,
-                                    near, status), "pr2_route_predict")
-        B.check(B.pr2_moe_forward(dm, x, ixd[b], gates, L["W_gate"], L["W_up"], L["W_down"],
-                                  L["Ws_gate"], L["Ws_up"], L["Ws_down"], o1[b], workspace=ws,
-                                  status=status), "pr2_moe_forward")
+        B.check(B.pr2_moe_rollout_forward(dm, x, L["W_router"], L["W_pred"], ixd[b], gates,
+                                          logits, near, L["W_gate"], L["W_up"], L["W_down"],
+                                          L["Ws_gate"], L["Ws_up"], L["Ws_down"], o1[b],
+                                          workspace=ws, status=status),
+                "pr2_moe_rollout_forward")
         B.check(B.pr2_moe_replay_forward(dm, x, W2, ixd[b], rgates, None, L["W_gate"], L["W_up"],
                                          L["W_down"], L["Ws_gate"], L["Ws_up"], L["Ws_down"],
                                          o2[b], workspace=ws, status=status),

@@ -150,6 +150,24 @@ pr2_status pr2_moe_forward(const pr2_dims* dims, const void* h, const int32_t* i
                            const pr2_stage_events* events, void* stream);
 
 /*
+ * Rollout-mode layer in one call: pr2_route_predict followed by pr2_moe_forward on the route
+ * and gates it records (Eqs. pr2_predict, pr2_route, pr2_old_output; Algorithm 2), with
+ * identical results.  On the tensor-core path the routing kernel also counts, per CTA, the
+ * experts of the rows it finishes into the workspace, so dispatch needs neither a histogram
+ * pass nor a grid-wide barrier and runs as an ordinary launch right behind the routing kernel.
+ * Arguments as in pr2_route_predict (idx, gates, logits_old, near_tie written) and
+ * pr2_moe_forward (the rest; the workspace is the same size).
+ */
+pr2_status pr2_moe_rollout_forward(const pr2_dims* dims, const void* h, const void* W_router,
+                                   const void* W_pred, int32_t* idx, float* gates,
+                                   float* logits_old, int64_t* near_tie, const void* W_gate,
+                                   const void* W_up, const void* W_down, const void* Ws_gate,
+                                   const void* Ws_up, const void* Ws_down, void* out,
+                                   int32_t* counts, int32_t* perm, void* workspace,
+                                   size_t ws_bytes, int32_t* status_dev,
+                                   const pr2_stage_events* events, void* stream);
+
+/*
  * Training-mode layer in one call: pr2_route_replay followed by pr2_moe_forward on its gates
  * (Sec. 4.1 "Replay During Training", Eq. pr2_output), with identical results.  Only the
  * gate-weighted combine reads the replay gates, so the call launches dispatch and the expert

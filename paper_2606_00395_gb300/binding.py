@@ -111,6 +111,10 @@ def load() -> ctypes.CDLL:
         lib.pr2_moe_replay_forward.argtypes = [D, P, P, P, P, P, P, P, P, P, P, P, P, P, P, P,
                                                ctypes.c_size_t, P, ctypes.POINTER(StageEvents), P]
         lib.pr2_moe_replay_forward.restype = ctypes.c_int
+        lib.pr2_moe_rollout_forward.argtypes = [D, P, P, P, P, P, P, P, P, P, P, P, P, P, P, P,
+                                                P, P, ctypes.c_size_t, P,
+                                                ctypes.POINTER(StageEvents), P]
+        lib.pr2_moe_rollout_forward.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -170,6 +174,21 @@ def pr2_moe_forward(dm: Dims, h, idx, gates, W_gate, W_up, W_down, Ws_gate, Ws_u
                                   _p(out), _p(counts), _p(perm), _p(workspace),
                                   ctypes.c_size_t(ws_bytes), _p(status),
                                   None if events is None else ctypes.byref(events), _s(stream))
+
+
+def pr2_moe_rollout_forward(dm: Dims, h, W_router, W_pred, idx, gates, logits_old, near_tie,
+                            W_gate, W_up, W_down, Ws_gate, Ws_up, Ws_down, out, counts=None,
+                            perm=None, workspace=None, ws_bytes=None, status=None,
+                            events: Optional[StageEvents] = None, stream=None) -> int:
+    """``pr2_route_predict`` then ``pr2_moe_forward`` in one call (route, gates, optional
+    logits and near-tie count written); dispatch reads the routing kernel's histograms."""
+    if ws_bytes is None:
+        ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    return load().pr2_moe_rollout_forward(
+        ctypes.byref(dm), _p(h), _p(W_router), _p(W_pred), _p(idx), _p(gates), _p(logits_old),
+        _p(near_tie), _p(W_gate), _p(W_up), _p(W_down), _p(Ws_gate), _p(Ws_up), _p(Ws_down),
+        _p(out), _p(counts), _p(perm), _p(workspace), ctypes.c_size_t(ws_bytes), _p(status),
+        None if events is None else ctypes.byref(events), _s(stream))
 
 
 def pr2_moe_replay_forward(dm: Dims, h, W_router, idx, gates, probs, W_gate, W_up, W_down,

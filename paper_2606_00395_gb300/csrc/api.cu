@@ -84,6 +84,7 @@ struct Workspace {
   TileEntry* tiles;
   TileEntry* stiles1;
   TileEntry* stiles2;
+  int32_t* route_hist;  // per-CTA expert histograms of the rollout routing (pr2_moe_rollout_forward)
   void* xperm;
   void* hbuf;
   void* ybuf;
@@ -119,9 +120,15 @@ Workspace carve(const pr2_dims& dm, uint8_t* base) {
   w.tiles = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * w.max_tiles));
   w.stiles1 = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * (w.shared_tiles + 1)));
   w.stiles2 = reinterpret_cast<TileEntry*>(take(sizeof(TileEntry) * (w.shared_tiles + 1)));
+
   // permuted copy of h: only the fp32 path reads it; the bf16 gate/up GEMM gathers from h
   w.xperm = dm.dtype == PR2_FP32 ? take(es * F * dm.d) : nullptr;
-  w.hbuf = take(es * F * dm.m);
+  // H [Tk, m].  The rollout routing's per-CTA histograms share its first bytes: dispatch reads
+  // them before the gate/up GEMM (which waits for dispatch) writes H.
+  const size_t hist_bytes = sizeof(int32_t) * (size_t)mt_T * kRouteMaxSplit * dm.N;
+  const size_t h_bytes = es * F * dm.m;
+  w.hbuf = take(h_bytes > hist_bytes ? h_bytes : hist_bytes);
+  w.route_hist = static_cast<int32_t*>(w.hbuf);
   w.ybuf = take(es * F * dm.d);
   w.hs = take(es * dm.n_shared * dm.T * dm.m);
   w.ys = take(es * dm.n_shared * dm.T * dm.d);
@@ -146,7 +153,8 @@ pr2_status finish(cudaError_t err, uint32_t flags, int32_t* status_dev, cudaStre
 pr2_status route_common(const pr2_dims* dims, bool predict, const void* h, const void* W,
                         const void* Wp, const int32_t* idx_in, int32_t* idx_out, float* gates,
                         float* aux, int64_t* near_tie, int32_t* status_dev, void* stream,
-                        bool late_wait = false) {
+                        bool late_wait = false, int32_t* hist = nullptr,
+                        int* split_out = nullptr) {
   pr2_status s = check_dims(dims);
   if (s != PR2_OK) return s;
   const pr2_dims& dm = *dims;
@@ -194,6 +202,8 @@ pr2_status route_common(const pr2_dims* dims, bool predict, const void* h, const
     a.norm = (dm.flags & PR2_F_NORMALIZE_TOPK) ? 1 : 0;
     a.compact = compact ? 1 : 0;
     a.late_wait = late_wait ? 1 : 0;
+    a.hist = predict ? hist : nullptr;
+    if (split_out != nullptr) *split_out = split;
     err = launch_route_tc(mode, tm_h, tm_w, tm_wp, a, split, st);
   }
   return finish(err, dm.flags, status_dev, st);
@@ -394,17 +404,11 @@ struct ReplayRoute {
 // alias `out`) is added to the combined output.  With `replay`, the replay gates of the route
 // `idx` are computed into `gates` after the expert GEMMs and before the combine, which is the
 // only step that reads them.
-pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* idx,
-                            const float* gates, const void* W_gate, const void* W_up,
-                            const void* W_down, const void* Ws_gate, const void* Ws_up,
-                            const void* Ws_down, void* out, const void* residual,
-                            int32_t* counts, int32_t* perm, void* workspace, size_t ws_bytes,
-                            int32_t* status_dev, const pr2_stage_events* events,
-                            void* stream, const ReplayRoute* replay = nullptr) {
-  pr2_status s = check_dims(dims);
-  if (s != PR2_OK) return s;
-  const pr2_dims& dm = *dims;
-  if (dm.T == 0) return PR2_OK;  // empty layer: nothing to write
+// Host-side checks of pr2_moe_forward's arguments (dims already checked, T > 0).
+pr2_status forward_args(const pr2_dims& dm, const void* h, const int32_t* idx, const float* gates,
+                        const void* W_gate, const void* W_up, const void* W_down,
+                        const void* Ws_gate, const void* Ws_up, const void* Ws_down, void* out,
+                        void* workspace, size_t ws_bytes) {
   if (h == nullptr || idx == nullptr || gates == nullptr || W_gate == nullptr ||
       W_up == nullptr || W_down == nullptr || out == nullptr)
     return PR2_ERR_INVALID_ARG;
@@ -421,6 +425,31 @@ pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* 
   if (workspace == nullptr || ws_bytes < probe.total ||
       (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return PR2_ERR_WORKSPACE;
+  return PR2_OK;
+}
+
+// Per-CTA expert histograms that the rollout routing kernel wrote for this layer's route
+// (pr2_moe_rollout_forward): dispatch then needs no histogram pass of its own.
+struct RouteHist {
+  const int32_t* hist;
+  int split;
+};
+
+pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* idx,
+                            const float* gates, const void* W_gate, const void* W_up,
+                            const void* W_down, const void* Ws_gate, const void* Ws_up,
+                            const void* Ws_down, void* out, const void* residual,
+                            int32_t* counts, int32_t* perm, void* workspace, size_t ws_bytes,
+                            int32_t* status_dev, const pr2_stage_events* events,
+                            void* stream, const ReplayRoute* replay = nullptr,
+                            const RouteHist* rhist = nullptr) {
+  pr2_status s = check_dims(dims);
+  if (s != PR2_OK) return s;
+  const pr2_dims& dm = *dims;
+  if (dm.T == 0) return PR2_OK;  // empty layer: nothing to write
+  s = forward_args(dm, h, idx, gates, W_gate, W_up, W_down, Ws_gate, Ws_up, Ws_down, out,
+                   workspace, ws_bytes);
+  if (s != PR2_OK) return s;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const Workspace w = carve(dm, static_cast<uint8_t*>(workspace));
   int32_t* status = status_dev ? status_dev : w.status;
@@ -441,7 +470,10 @@ pr2_status moe_forward_impl(const pr2_dims* dims, const void* h, const int32_t* 
                   w.stiles1, w.stiles2,  h,         w.xperm, status, w.sync_ctr,
                   dm.dtype == PR2_BF16 ? w.ready : nullptr, kTileM};
   // (w.xperm is nullptr on the bf16 path: dispatch then launches no gather)
-  if (err == cudaSuccess) err = launch_dispatch(da, num_sms, st);
+  if (err == cudaSuccess)
+    err = (rhist != nullptr && dm.dtype == PR2_BF16)
+              ? launch_dispatch_from_hist(da, rhist->hist, rhist->split, st)
+              : launch_dispatch(da, num_sms, st);
   mark(events ? events->dispatched : nullptr);
   if (err != cudaSuccess) return PR2_ERR_CUDA;
 
@@ -536,6 +568,47 @@ pr2_status pr2_moe_forward(const pr2_dims* dims, const void* h, const int32_t* i
   return moe_forward_impl(dims, h, idx, gates, W_gate, W_up, W_down, Ws_gate, Ws_up, Ws_down,
                           out, nullptr, counts, perm, workspace, ws_bytes, status_dev, events,
                           stream);
+}
+
+pr2_status pr2_moe_rollout_forward(const pr2_dims* dims, const void* h, const void* W_router,
+                                   const void* W_pred, int32_t* idx, float* gates,
+                                   float* logits_old, int64_t* near_tie, const void* W_gate,
+                                   const void* W_up, const void* W_down, const void* Ws_gate,
+                                   const void* Ws_up, const void* Ws_down, void* out,
+                                   int32_t* counts, int32_t* perm, void* workspace,
+                                   size_t ws_bytes, int32_t* status_dev,
+                                   const pr2_stage_events* events, void* stream) {
+  pr2_status s = check_dims(dims);
+  if (s != PR2_OK) return s;
+  const pr2_dims& dm = *dims;
+  if (dm.T == 0) return PR2_OK;
+  if ((dm.flags & PR2_F_SYNC_STATUS) && status_dev == nullptr) return PR2_ERR_INVALID_ARG;
+  // everything both steps need is checked before anything is launched
+  if (W_router == nullptr || W_pred == nullptr || !aligned16(W_router) || !aligned16(W_pred) ||
+      (logits_old != nullptr && !aligned16(logits_old)))
+    return PR2_ERR_INVALID_ARG;
+  s = forward_args(dm, h, idx, gates, W_gate, W_up, W_down, Ws_gate, Ws_up, Ws_down, out,
+                   workspace, ws_bytes);
+  if (s != PR2_OK) return s;
+  pr2_dims dr = dm;
+  dr.flags &= ~PR2_F_SYNC_STATUS;
+  if (dm.dtype != PR2_BF16) {  // fp32: the two calls in sequence
+    s = route_common(&dr, true, h, W_router, W_pred, nullptr, idx, gates, logits_old, near_tie,
+                     status_dev, stream);
+    if (s != PR2_OK) return s;
+    return moe_forward_impl(dims, h, idx, gates, W_gate, W_up, W_down, Ws_gate, Ws_up, Ws_down,
+                            out, nullptr, counts, perm, workspace, ws_bytes, status_dev, events,
+                            stream);
+  }
+  const Workspace w = carve(dm, static_cast<uint8_t*>(workspace));
+  int split = 1;
+  s = route_common(&dr, true, h, W_router, W_pred, nullptr, idx, gates, logits_old, near_tie,
+                   status_dev, stream, false, w.route_hist, &split);
+  if (s != PR2_OK) return s;
+  const RouteHist rh{w.route_hist, split};
+  return moe_forward_impl(dims, h, idx, gates, W_gate, W_up, W_down, Ws_gate, Ws_up, Ws_down,
+                          out, nullptr, counts, perm, workspace, ws_bytes, status_dev, events,
+                          stream, nullptr, &rh);
 }
 
 pr2_status pr2_moe_replay_forward(const pr2_dims* dims, const void* h, const void* W_router,

@@ -425,6 +425,128 @@ __global__ void __launch_bounds__(kDispatchChunk)
   }
 }
 
+// Dispatch of a route that the routing kernel just wrote, from its per-CTA histograms: block b
+// handles the slots of routing tile b (128 tokens x k slots, one thread per slot).  Every block
+// derives the expert totals and its own prefix from the histogram rows (int4 column reads),
+// then places its slots in stable order exactly as dispatch_fused_kernel does; block 0 writes
+// counts, offsets and the tile tables.  Every slot is valid (the routing kernel wrote k distinct
+// experts in [0, N) per token), which is what the histograms counted.
+constexpr int kHistBlock = kTileM * kMaxTopK;  // 1024 threads: the slots of one routing tile
+constexpr int kHistWarps = kHistBlock / 32;
+
+__global__ void __launch_bounds__(kHistBlock)
+    dispatch_hist_kernel(const int32_t* __restrict__ idx, int64_t T, int k, int N, int n_shared,
+                         int tile_rows, const int32_t* __restrict__ hist, int hist_rows,
+                         int split, int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
+                         int32_t* __restrict__ perm, int32_t* __restrict__ inv,
+                         TileEntry* __restrict__ tiles, int32_t* __restrict__ num_tiles,
+                         TileEntry* __restrict__ stiles1, TileEntry* __restrict__ stiles2,
+                         int32_t* __restrict__ ready) {
+  extern __shared__ int dsm[];
+  int* wcnt = dsm;                     // [kHistWarps][N] per-warp counts, then per-warp bases
+  int* tot = wcnt + kHistWarps * N;    // [N]
+  int* pre = tot + N;                  // [N] slots of each expert in earlier tiles
+  int* ex_off = pre + N;               // [N+1]
+  int* ex_tile = ex_off + N + 1;       // [N+1]
+  __shared__ int sh[32];
+  const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31;
+  const int b = static_cast<int>(blockIdx.x);
+  for (int i = tid; i < kHistWarps * N; i += kHistBlock) wcnt[i] = 0;
+  for (int i = tid; i < N; i += kHistBlock) {
+    tot[i] = 0;
+    pre[i] = 0;
+  }
+  pdl_wait();  // the route and its histograms come from the routing kernel
+  pdl_trigger();
+  __syncthreads();
+  // ---- expert totals and this tile's prefix: hist rows [0, hist_rows), before = rows < b*split
+  const int n4 = N / 4, G = kHistBlock / n4;
+  const int q = tid % n4, g = tid / n4;
+  const int before_rows = b * split;
+  if (g < G) {
+    int4 all = make_int4(0, 0, 0, 0), bef = make_int4(0, 0, 0, 0);
+    const int4* col = reinterpret_cast<const int4*>(hist) + q;
+    for (int r0 = g; r0 < hist_rows; r0 += 8 * G) {
+      int4 v[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int r = r0 + j * G;
+        v[j] = r < hist_rows ? __ldcg(col + static_cast<int64_t>(r) * n4) : make_int4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int r = r0 + j * G;
+        all.x += v[j].x;
+        all.y += v[j].y;
+        all.z += v[j].z;
+        all.w += v[j].w;
+        if (r < before_rows) {
+          bef.x += v[j].x;
+          bef.y += v[j].y;
+          bef.z += v[j].z;
+          bef.w += v[j].w;
+        }
+      }
+    }
+    atomicAdd(&tot[4 * q], all.x);
+    atomicAdd(&tot[4 * q + 1], all.y);
+    atomicAdd(&tot[4 * q + 2], all.z);
+    atomicAdd(&tot[4 * q + 3], all.w);
+    atomicAdd(&pre[4 * q], bef.x);
+    atomicAdd(&pre[4 * q + 1], bef.y);
+    atomicAdd(&pre[4 * q + 2], bef.z);
+    atomicAdd(&pre[4 * q + 3], bef.w);
+  }
+  // ---- this tile's slots: per-warp counts
+  const int64_t F = T * k;
+  const int64_t f = static_cast<int64_t>(b) * kTileM * k + tid;
+  const bool own = tid < kTileM * k && f < F;
+  const int e = own ? idx[f] : -1;
+  const unsigned same = __match_any_sync(0xffffffffu, e);
+  if (e >= 0 && lane == __ffs(same) - 1) wcnt[w * N + e] = __popc(same);
+  __syncthreads();
+  int all_rows, all_tiles;
+  const int total = tid < N ? tot[tid] : 0;
+  const int off = block_exclusive_scan(total, sh, &all_rows);
+  const int tstart =
+      block_exclusive_scan(tid < N ? (total + tile_rows - 1) / tile_rows : 0, sh, &all_tiles);
+  if (tid < N) {
+    ex_off[tid] = off;
+    ex_tile[tid] = tstart;
+  }
+  if (tid == 0) {
+    ex_off[N] = all_rows;
+    ex_tile[N] = all_tiles;
+  }
+  __syncthreads();
+  if (b == 0) {
+    if (tid < N) {
+      counts[tid] = total;
+      offsets[tid] = off;
+    }
+    if (tid == 0) offsets[N] = all_rows;
+    write_tile_tables(N, T, n_shared, tile_rows, ex_off, ex_tile, tiles, num_tiles, stiles1,
+                      stiles2, ready);
+  }
+  // ---- stable placement: per-warp bases, then ranks within the warp
+  for (int x = tid; x < N; x += kHistBlock) {
+    int run = ex_off[x] + pre[x];
+    for (int ww = 0; ww < kHistWarps; ++ww) {
+      const int c = wcnt[ww * N + x];
+      wcnt[ww * N + x] = run;
+      run += c;
+    }
+  }
+  __syncthreads();
+  if (own) {
+    const int pos = wcnt[w * N + e] + __popc(same & lanemask_lt());
+    perm[pos] = static_cast<int32_t>(f);
+    inv[f] = pos;
+  }
+}
+
+size_t hist_smem_bytes(int N) { return sizeof(int) * (static_cast<size_t>(kHistWarps) * N + 4 * N + 2); }
+
 size_t fused_smem_bytes(int N) { return sizeof(int) * (static_cast<size_t>(kWarps) * N + 4 * N + 2); }
 
 // Whether the fused dispatch can run (shape, and every block resident at once), cached per
@@ -770,6 +892,22 @@ cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st)
     if (err != cudaSuccess) return err;
   }
   return cudaSuccess;
+}
+
+cudaError_t launch_dispatch_from_hist(const DispatchArgs& a, const int32_t* hist, int split,
+                                      cudaStream_t st) {
+  const int tiles_r = static_cast<int>((a.T + kTileM - 1) / kTileM);
+  if (tiles_r == 0) return cudaSuccess;
+  if (a.N % 4 != 0 || a.k > kMaxTopK || hist == nullptr || split < 1) return cudaErrorInvalidValue;
+  const size_t smem = hist_smem_bytes(a.N);
+  cudaError_t err = cudaFuncSetAttribute(dispatch_hist_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+  if (err != cudaSuccess) return err;
+  return launch_pdl(dispatch_hist_kernel, dim3(tiles_r), dim3(kHistBlock), smem, st, 1, a.idx,
+                    a.T, a.k, a.N, a.n_shared, a.tile_rows, hist, tiles_r * split, split,
+                    a.counts, a.offsets, a.perm, a.inv, a.tiles, a.num_tiles, a.stiles1,
+                    a.stiles2, a.ready);
 }
 
 cudaError_t launch_combine(const CombineArgs& a, int num_sms, cudaStream_t st) {

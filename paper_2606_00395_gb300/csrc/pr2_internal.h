@@ -49,6 +49,7 @@ constexpr int kMaxTopK = 8;         // slots kept by the tensor-core routing epi
 constexpr int kMaxTopKSimt = 32;    // slots of the fp32 SIMT routing kernel
 constexpr int kMaxExperts = 256;    // routed experts supported by the routing kernels
 constexpr int kMaxExpertsDispatch = 1024;
+constexpr int kRouteMaxSplit = 8;   // most CTAs splitting one routing tile (histogram rows)
 
 // ---- routing (route_simt.cu, route_tc.cu) -------------------------------------------------
 cudaError_t launch_route_simt(const pr2_dims& dm, bool predict, const float* h, const float* W,
@@ -75,6 +76,8 @@ struct RouteTcArgs {
   int compact;             // 1: half the pipeline stages, so two CTAs share an SM (split 1)
   int late_wait;           // 1: the inputs are known ready; wait for the previous kernel only
                            // before exiting (the launch overlaps it; see pr2_moe_replay_forward)
+  int32_t* hist;           // predict, nullable: [CTAs][N] experts of each CTA's finished rows
+                           // (CTA tile * split + rank), read by dispatch_from_hist
   // kModeLoss only (h = h_old, W = W_p)
   const float* p_old;      // [T, N] cached router logits
   const float* rho;        // [T_rho, N] teacher probabilities
@@ -118,6 +121,11 @@ struct DispatchArgs {
   int tile_rows;           // most rows of one routed tile (an expert's rows are split evenly)
 };
 cudaError_t launch_dispatch(const DispatchArgs& a, int num_sms, cudaStream_t st);
+// Dispatch of a route the routing kernel just wrote (every slot valid), from the per-CTA
+// expert histograms it wrote: hist rows [tile * split + r], `split` rows per 128-token tile.
+// No histogram pass and no grid barrier, so it is an ordinary launch behind the routing kernel.
+cudaError_t launch_dispatch_from_hist(const DispatchArgs& a, const int32_t* hist, int split,
+                                      cudaStream_t st);
 
 struct CombineArgs {
   const void* Y;        // [T*k, d] expert outputs in dispatch order

@@ -43,6 +43,7 @@ constexpr int kBK = 64;                          // bf16 elements per 128-byte s
 constexpr int kATileBytes = kTileM * kBK * 2;    // 16 KB
 constexpr int kKeep = kMaxTopK + 1;              // top-(k+1) kept for the margin
 constexpr int kMaxSplit = 8;
+static_assert(kMaxSplit == kRouteMaxSplit, "histogram rows per routing tile");
 constexpr int kMaxStages = 12;
 constexpr int kStageBudget = 192 * 1024;    // pipeline stages of a CTA alone on its SM
 constexpr int kCompactBudget = 96 * 1024;   // two CTAs per SM (more token tiles than SMs)
@@ -295,6 +296,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // ---------------- epilogue ----------------
   const bool epi = warp >= 2;
+  // predict: experts of the rows this CTA finishes, for the dispatch that follows
+  __shared__ int hist_s[kMaxExperts];
+  const bool count = predict && a.hist != nullptr;
+  if (count && epi) {
+    for (int e = threadIdx.x - 64; e < N; e += 128) hist_s[e] = 0;
+    named_bar_sync(1, 128);
+  }
   const int q = warp & 3;
   const int row = q * 32 + lane;  // TMEM lane of this thread
   const uint32_t trow = tmem + (static_cast<uint32_t>(q * 32) << 16);
@@ -475,7 +483,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           other[j] = j < kKeep ? __shfl_xor_sync(0xffffffffu, top[j], o) : 0ull;
         merge16_desc(top, other);
       }
-      if (have && live && part == 0) tie = predict_write(top, mx, inv_s, t, a);
+      if (have && live && part == 0) {
+        tie = predict_write(top, mx, inv_s, t, a);
+        if (count)
+          for (int j = 0; j < k; ++j) atomicAdd(&hist_s[key_e(top[j])], 1);
+      }
     } else if (!loss) {
       // Each valid slot's z is held by the one thread owning its expert; the others hold 0.
 #pragma unroll
@@ -518,6 +530,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0 && ties != 0u && a.near_tie != nullptr)
       atomicAdd(reinterpret_cast<unsigned long long*>(a.near_tie),
                 static_cast<unsigned long long>(__popc(ties)));
+    if (count) {  // every row of this CTA counted: publish its histogram row (zeros included)
+      named_bar_sync(1, 128);
+      int32_t* hrow = a.hist + static_cast<int64_t>(blockIdx.x) * N;
+      for (int e = threadIdx.x - 64; e < N; e += 128) hrow[e] = hist_s[e];
+    }
     tc_fence_before();
   }
   if (epi && loss) {

@@ -312,3 +312,39 @@ def test_replay_layer_call_equals_the_two_calls(name):
     want_status = int(r["status"].item()) | int(ref["status"].item())
     assert int(status.item()) == want_status
     assert (want_status & B.PR2_STATUS_BAD_INDEX) == (B.PR2_STATUS_BAD_INDEX if cfg.T > 3 else 0)
+
+
+@pytest.mark.parametrize("name", ["tiny_fp32", "bf16_fused_dispatch", "bf16_multitile",
+                                  "bf16_partial_n", "bf16_shared_n256", "bf16_top1",
+                                  "bf16_one_token"])
+def test_rollout_layer_call_equals_the_two_calls(name):
+    """pr2_moe_rollout_forward (dispatch from the routing kernel's per-CTA histograms) writes
+    exactly what pr2_route_predict followed by pr2_moe_forward writes: route, gates, logits,
+    near-tie count, counts, permutation and layer output, bit for bit."""
+    cfg = SMALL[name]
+    L = synth.make_layer(cfg, seed=12)
+    Ld = H.to_dev(L)
+    g = H.gpu_predict(cfg, Ld)
+    ref = H.gpu_forward(cfg, Ld, g["idx"], g["gates"])
+    assert ref["code"] == 0
+    dm = H.dims_of(cfg)
+    idx = torch.full_like(g["idx"], -7)
+    gates = torch.full_like(g["gates"], float("nan"))
+    logits = torch.full_like(g["logits"], float("nan"))
+    near = torch.zeros(1, dtype=torch.int64, device="cuda")
+    out = torch.full_like(ref["out"], float("nan"))
+    counts = torch.full_like(ref["counts"], -1)
+    perm = torch.full_like(ref["perm"], -1)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    code = B.pr2_moe_rollout_forward(dm, Ld["x"], Ld["W_router"], Ld["W_pred"], idx, gates,
+                                     logits, near, Ld["W_gate"], Ld["W_up"], Ld["W_down"],
+                                     Ld["Ws_gate"], Ld["Ws_up"], Ld["Ws_down"], out,
+                                     counts=counts, perm=perm, workspace=B.alloc_workspace(dm),
+                                     status=status)
+    assert code == 0, B.pr2_strerror(code)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    assert torch.equal(idx, g["idx"]) and torch.equal(gates, g["gates"])
+    assert torch.equal(logits, g["logits"]) and torch.equal(near, g["near_tie"])
+    assert torch.equal(counts, ref["counts"]) and torch.equal(perm, ref["perm"])
+    assert torch.equal(out, ref["out"])
