@@ -215,7 +215,7 @@ struct LossWorkspace {
   uint16_t* gt;     // bf16: [N, Tpad] dKL/dz transposed
   float* G;         // fp32: [Tc, N] dKL/dz
   float* kl;        // [Tpad] per-token KL when the caller passes none
-  float* partial;   // bf16: [kLossMaxSplit, N, d]
+  float* partial;   // bf16: split partial tiles of the gradient, [kLossMaxSplit, Npad, dpad]
   int Tpad;
   size_t total;
 };
@@ -234,7 +234,7 @@ LossWorkspace carve_loss(const pr2_dims& dm, uint8_t* base) {
   if (dm.dtype == PR2_BF16) {
     w.gt = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * (size_t)dm.N * w.Tpad));
     w.partial = reinterpret_cast<float*>(
-        take(sizeof(float) * (size_t)kLossMaxSplit * dm.N * (size_t)dm.d));
+        take(sizeof(float) * (size_t)kLossMaxSplit * loss_grad_rows(dm.N) * loss_grad_cols(dm.d)));
   } else {
     w.G = reinterpret_cast<float*>(take(sizeof(float) * (size_t)dm.T * dm.N));
   }
@@ -303,7 +303,7 @@ pr2_status pr2_predictor_loss(const pr2_dims* dims, const void* h_old, const flo
   const int Tc = static_cast<int>(dm.T);
   float* kl = kl_tok ? kl_tok : w.kl;
   const int delta = (dm.flags & PR2_F_DELTA_LOSS) ? 1 : 0;
-  GradArgs g{dm.N, dm.d, Tc, w.Tpad, 1, nullptr, grad_Wp, kl, loss, status};
+  GradArgs g{dm.N, dm.d, Tc, w.Tpad, 1, w.partial, grad_Wp, kl, loss, status};
   if (dm.dtype == PR2_FP32) {
     err = launch_loss_simt(static_cast<const float*>(h_old), p_old,
                            static_cast<const float*>(W_pred), rho, T_rho, pos, delta, Tc, dm.d,
@@ -339,9 +339,7 @@ pr2_status pr2_predictor_loss(const pr2_dims* dims, const void* h_old, const flo
   const int split = route_split(Tc, dm.N, dm.d, kModeLoss, num_sms);
   err = launch_route_tc(kModeLoss, tm_h, tm_w, tm_w, a, split, st);
   g.split = loss_grad_split(dm.N, dm.d, w.Tpad, num_sms);
-  g.partial = w.partial;
   if (err == cudaSuccess) err = launch_loss_grad_tc(tm_gt, tm_hmn, g, st);
-  if (err == cudaSuccess) err = launch_loss_finish(g, st);
   return finish(err, dm.flags, status_dev, st);
 }
 

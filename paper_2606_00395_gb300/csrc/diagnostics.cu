@@ -1,7 +1,7 @@
 // Route-tracking diagnostics (Sec. 5 "Top-k Agreement and Route KL", "Deviation Tails") and the
 // fixed-length feature-cache writer (Algorithm 2, App. "uniform sub-sampling").
 //
-// Diagnostics: one warp per token.  Lane l holds rho[t, 32 j + l].  A cached expert e lies in
+// Diagnostics: one warp per token.  Lane l holds rho[t, 32 j + l] and cached slot l.  A cached expert e lies in
 // I_t = TopK(rho_t, k) (largest values, the lower expert first on equal values, as TopK of Eq.
 // pr2_route) exactly when fewer than k experts beat it, where j beats e if rho_j > rho_e or
 // rho_j = rho_e and j < e; the warp counts the experts that beat each cached entry with ballots.
@@ -36,6 +36,9 @@ __global__ void __launch_bounds__(kWarps * 32)
   for (int64_t t = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5); t < T;
        t += nwarps) {
     const float* row = rho + t * N;
+    // One round of loads per token: the row of rho and the k cached entries (lane sl holds
+    // slot sl), so that nothing below waits on a dependent global load.
+    const int e_l = lane < k ? cached[t * k + lane] : -1;
     float v[kPerLane];
 #pragma unroll
     for (int j = 0; j < kPerLane; ++j) {
@@ -43,14 +46,27 @@ __global__ void __launch_bounds__(kWarps * 32)
       v[j] = e < N ? row[e] : 0.f;
     }
     const int nj = (N + 31) / 32;
+    // slot sl counts if its entry is in range and no earlier slot holds the same expert
+    bool ok_l = lane < k && e_l >= 0 && e_l < N;
+    for (int s2 = 0; s2 < k - 1; ++s2) {
+      const int es = __shfl_sync(0xffffffffu, e_l, s2);
+      if (s2 < lane && es == e_l) ok_l = false;
+    }
+    // rho[t, e_l] fetched from the lane that holds it
+    const int src = ok_l ? e_l : 0;
+    float re_l = 0.f;
+#pragma unroll
+    for (int j = 0; j < kPerLane; ++j) {
+      if (j >= nj) break;
+      const float x = __shfl_sync(0xffffffffu, v[j], src & 31);
+      if (j == (src >> 5)) re_l = x;
+    }
+    const unsigned okmask = __ballot_sync(0xffffffffu, ok_l);
     int ov = 0;
     for (int sl = 0; sl < k; ++sl) {  // uniform over the warp
-      const int e = cached[t * k + sl];
-      bool ok = e >= 0 && e < N;
-      for (int s2 = 0; ok && s2 < sl; ++s2)
-        if (cached[t * k + s2] == e) ok = false;
-      if (!ok) continue;
-      const float re = row[e];
+      const int e = __shfl_sync(0xffffffffu, e_l, sl);
+      const float re = __shfl_sync(0xffffffffu, re_l, sl);
+      if (!((okmask >> sl) & 1u)) continue;
       int beat = 0;
 #pragma unroll
       for (int j = 0; j < kPerLane; ++j) {
@@ -88,7 +104,20 @@ __global__ void __launch_bounds__(256)
     if (lane == 0) pos[c] = static_cast<int32_t>(p);
     const uint4* src = h + p * row_vec;
     uint4* dst = cache_h + c * row_vec;
-    for (int v = lane; v < row_vec; v += 32) dst[v] = __ldg(src + v);
+    // eight 16-byte loads in flight per lane before the stores (a 4 KB row in one round)
+    for (int v0 = 0; v0 < row_vec; v0 += 8 * 32) {
+      uint4 r[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int v = v0 + j * 32 + lane;
+        if (v < row_vec) r[j] = __ldg(src + v);
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int v = v0 + j * 32 + lane;
+        if (v < row_vec) dst[v] = r[j];
+      }
+    }
     if (logits != nullptr) {
       const float* ls = logits + p * N;
       float* ld = cache_p + c * N;

@@ -326,6 +326,11 @@ __device__ __forceinline__ void reg_fence(uint32_t (&r)[16]) {
 }
 
 // ------------------------------------------------------------------------------------------
+// Barrier `id` (1-15) over `count` threads (a multiple of 32) of this CTA.
+__device__ __forceinline__ void named_bar_sync(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 // Thread-block clusters and distributed shared memory.
 // ------------------------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t cluster_ctarank() {

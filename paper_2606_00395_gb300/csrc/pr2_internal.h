@@ -182,8 +182,8 @@ cudaError_t launch_expert_simt(bool swiglu, const float* A, const float* Wb0, co
 // `partial` [split, N, d] fp32, then a fixed-order reduction.  fp32: SIMT kernels.
 struct GradArgs {
   int N, d, Tc, Tpad;
-  int split;              // token-block split of the GEMM
-  float* partial;         // [split, N, d]
+  int split;              // token-block split of the GEMM: CTAs per cluster (1, 2, 4 or 8)
+  float* partial;         // [split, N, d] fp32 split partials (split > 1)
   float* grad;            // [N, d]
   const float* kl_tok;    // [Tc]
   float* loss;            // [1]
@@ -191,8 +191,12 @@ struct GradArgs {
 };
 constexpr int kLossMaxSplit = 8;
 int loss_grad_split(int N, int d, int Tpad, int num_sms);
+// Rows (experts) and columns (d) of the gradient rounded up to whole output tiles.
+int64_t loss_grad_rows(int N);
+int64_t loss_grad_cols(int d);
 cudaError_t launch_loss_grad_tc(const CUtensorMap& tm_gt, const CUtensorMap& tm_h,
                                 const GradArgs& g, cudaStream_t st);
+// fp32 path: the loss from the per-token KL (the bf16 gradient kernel sums it itself).
 cudaError_t launch_loss_finish(const GradArgs& g, cudaStream_t st);
 // fp32 path: per-token KL and G [Tc, N] (row-major), then the gradient.
 cudaError_t launch_loss_simt(const float* h_old, const float* p_old, const float* Wp,

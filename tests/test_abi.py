@@ -118,7 +118,7 @@ def test_predictor_loss_rejects_bad_arguments_on_the_host(lib):
     fake = ctypes.c_void_p(256)
     ws = B.pr2_predictor_loss_workspace_bytes(dm)
     assert ws > 0
-    # bf16 workspace holds dKL/dz (N x T_c) and the split-K gradient partials
+    # bf16 workspace holds dKL/dz transposed (N x T_c) and the split-K gradient partials
     assert ws >= 128 * 256 * 2 + 8 * 128 * 2048 * 4
     ok = [ctypes.byref(dm), fake, fake, fake, fake, ctypes.c_int64(256), None, fake, None, fake]
     # missing output / input pointers
