@@ -1,25 +1,37 @@
 // Route-tracking diagnostics (Sec. 5 "Top-k Agreement and Route KL", "Deviation Tails") and the
 // fixed-length feature-cache writer (Algorithm 2, App. "uniform sub-sampling").
 //
-// Diagnostics: one warp per token.  Lane l holds rho[t, 32 j + l] and cached slot l.  A cached expert e lies in
-// I_t = TopK(rho_t, k) (largest values, the lower expert first on equal values, as TopK of Eq.
-// pr2_route) exactly when fewer than k experts beat it, where j beats e if rho_j > rho_e or
-// rho_j = rho_e and j < e; the warp counts the experts that beat each cached entry with ballots.
-// overlap_t = |Î_t ∩ I_t| counts the cached entries (in range, not repeated) that pass.  hist[k - overlap_t] and sum_t overlap_t are accumulated per block in shared memory
-// and then with 64-bit integer atomics (order-independent, so exact and deterministic); the
+// Diagnostics: one warp per token.  Lane l holds rho[t, 32 j + l] and cached slot l.  A cached
+// expert e lies in I_t = TopK(rho_t, k) (largest values, the lower expert first on equal
+// values, as TopK of Eq. pr2_route) exactly when fewer than k experts beat it, where j beats e
+// if rho_j > rho_e or rho_j = rho_e and j < e, i.e. if j's 64-bit rank key (orderable value
+// bits, inverted index) is larger; the warp counts the experts that beat each cached entry
+// with one ballot per 32 experts.
+// overlap_t = |Î_t ∩ I_t| counts the cached entries (in range, not repeated) that pass.
+// hist[k - overlap_t] and sum_t overlap_t are accumulated per block in shared memory and then
+// with 64-bit integer atomics (order-independent, so exact and deterministic); the
 // grid is at most two blocks per SM, each looping over tokens, so that the k + 2 global
 // counters see few atomics.
 // Feature cache: row c of the cache is row pos_c = floor(c T / T_c) of the batch; one warp per
-// cached row copies h (16-byte vectors) and the fp32 router logits.
+// cached row copies h (16-byte vectors, eight in flight per lane) and the fp32 router logits.
 #include "pr2_device.cuh"
 #include "pr2_internal.h"
 
 namespace pr2 {
 namespace {
 
-constexpr int kPerLane = kMaxExperts / 32;
 constexpr int kWarps = 16;
 
+// Rank key of expert e with probability x: a larger key ranks higher (larger x; on equal x the
+// lower expert).  -0 is taken as +0, so that equal values compare equal as floats do.
+__device__ __forceinline__ uint64_t rank_key(float x, int e) {
+  const uint32_t u = __float_as_uint(x + 0.0f);
+  const uint32_t ord = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  return (static_cast<uint64_t>(ord) << 32) | static_cast<uint32_t>(~e);
+}
+
+// kNJ = experts per lane (N <= 32 kNJ).
+template <int kNJ>
 __global__ void __launch_bounds__(kWarps * 32)
     diagnostics_kernel(const float* __restrict__ rho, const int32_t* __restrict__ cached,
                        int64_t T, int N, int k, unsigned long long* __restrict__ hist,
@@ -39,42 +51,38 @@ __global__ void __launch_bounds__(kWarps * 32)
     // One round of loads per token: the row of rho and the k cached entries (lane sl holds
     // slot sl), so that nothing below waits on a dependent global load.
     const int e_l = lane < k ? cached[t * k + lane] : -1;
-    float v[kPerLane];
+    float v[kNJ];
 #pragma unroll
-    for (int j = 0; j < kPerLane; ++j) {
+    for (int j = 0; j < kNJ; ++j) {
       const int e = j * 32 + lane;
       v[j] = e < N ? row[e] : 0.f;
     }
-    const int nj = (N + 31) / 32;
+    uint64_t key[kNJ];  // experts beyond N get key 0, below every real key
+#pragma unroll
+    for (int j = 0; j < kNJ; ++j) key[j] = j * 32 + lane < N ? rank_key(v[j], j * 32 + lane) : 0ull;
     // slot sl counts if its entry is in range and no earlier slot holds the same expert
     bool ok_l = lane < k && e_l >= 0 && e_l < N;
     for (int s2 = 0; s2 < k - 1; ++s2) {
       const int es = __shfl_sync(0xffffffffu, e_l, s2);
       if (s2 < lane && es == e_l) ok_l = false;
     }
-    // rho[t, e_l] fetched from the lane that holds it
+    // the rank key of this lane's slot, from the lane that holds rho[t, e_l]
     const int src = ok_l ? e_l : 0;
-    float re_l = 0.f;
+    uint64_t ks_l = 0;
 #pragma unroll
-    for (int j = 0; j < kPerLane; ++j) {
-      if (j >= nj) break;
-      const float x = __shfl_sync(0xffffffffu, v[j], src & 31);
-      if (j == (src >> 5)) re_l = x;
+    for (int j = 0; j < kNJ; ++j) {
+      const uint64_t x = __shfl_sync(0xffffffffu, key[j], src & 31);
+      if (j == (src >> 5)) ks_l = x;
     }
     const unsigned okmask = __ballot_sync(0xffffffffu, ok_l);
+    // a cached expert is in TopK(rho_t, k) iff fewer than k experts rank above it
     int ov = 0;
     for (int sl = 0; sl < k; ++sl) {  // uniform over the warp
-      const int e = __shfl_sync(0xffffffffu, e_l, sl);
-      const float re = __shfl_sync(0xffffffffu, re_l, sl);
+      const uint64_t ks = __shfl_sync(0xffffffffu, ks_l, sl);
       if (!((okmask >> sl) & 1u)) continue;
       int beat = 0;
 #pragma unroll
-      for (int j = 0; j < kPerLane; ++j) {
-        if (j >= nj) break;
-        const int ej = j * 32 + lane;
-        const bool b = ej < N && (v[j] > re || (v[j] == re && ej < e));
-        beat += __popc(__ballot_sync(0xffffffffu, b));
-      }
+      for (int j = 0; j < kNJ; ++j) beat += __popc(__ballot_sync(0xffffffffu, key[j] > ks));
       ov += beat < k ? 1 : 0;
     }
     if (lane == 0) {
@@ -135,9 +143,13 @@ cudaError_t launch_diagnostics(const float* rho, const int32_t* cached, int64_t 
   int64_t want = (T + kWarps - 1) / kWarps;
   if (want > 2 * static_cast<int64_t>(num_sms)) want = 2 * static_cast<int64_t>(num_sms);
   const unsigned blocks = static_cast<unsigned>(want);
-  return launch_pdl(diagnostics_kernel, dim3(blocks), dim3(kWarps * 32), 0, st, 1, rho, cached,
-                    T, N, k, reinterpret_cast<unsigned long long*>(hist),
-                    reinterpret_cast<unsigned long long*>(overlap_sum));
+  auto* h64 = reinterpret_cast<unsigned long long*>(hist);
+  auto* o64 = reinterpret_cast<unsigned long long*>(overlap_sum);
+  const dim3 grid(blocks), block(kWarps * 32);
+  if (N <= 32) return launch_pdl(diagnostics_kernel<1>, grid, block, 0, st, 1, rho, cached, T, N, k, h64, o64);
+  if (N <= 64) return launch_pdl(diagnostics_kernel<2>, grid, block, 0, st, 1, rho, cached, T, N, k, h64, o64);
+  if (N <= 128) return launch_pdl(diagnostics_kernel<4>, grid, block, 0, st, 1, rho, cached, T, N, k, h64, o64);
+  return launch_pdl(diagnostics_kernel<8>, grid, block, 0, st, 1, rho, cached, T, N, k, h64, o64);
 }
 
 cudaError_t launch_feature_cache(const void* h, const float* logits, int64_t T, int64_t Tc,
