@@ -51,6 +51,8 @@ constexpr int kCompactBudget = 96 * 1024;   // two CTAs per SM (more token tiles
 struct RouteSmemLayout {
   int stages;
   int b_rows;        // rows of the weight tile: 2N (predict) or N (replay)
+  int passes;        // passes over K: 2 streams [W] then [W_p] (predict, N > 128), else 1
+  int pass_rows;     // weight rows of a stage: b_rows / passes
   int stage_bytes;   // A + B
   int bar_offset;    // after all stages
   int total;         // dynamic smem bytes requested (incl. 1 KB alignment slack)
@@ -59,7 +61,12 @@ struct RouteSmemLayout {
 __host__ __device__ inline RouteSmemLayout route_layout(int N, bool predict, bool compact) {
   RouteSmemLayout L;
   L.b_rows = predict ? 2 * N : N;
-  L.stage_bytes = kATileBytes + L.b_rows * kBK * 2;
+  // Predict with more than 128 experts: [W; W_p] would make 80 KB stages (two in flight at
+  // most), so the router and the predictor weights stream in two passes over K instead, each
+  // stage holding N weight rows; h is read twice, but four stages overlap loads and MMAs.
+  L.passes = (L.b_rows > 256 && N % 32 == 0) ? 2 : 1;
+  L.pass_rows = L.b_rows / L.passes;
+  L.stage_bytes = kATileBytes + L.pass_rows * kBK * 2;
   L.stages = (compact ? kCompactBudget : kStageBudget) / L.stage_bytes;
   if (L.stages > kMaxStages) L.stages = kMaxStages;
   if (L.stages < 2) L.stages = 2;
@@ -191,9 +198,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int R = kTileM / split;             // rows finished by this CTA
   const int nr = N / split;                 // experts of one finishing thread
   const int nb4 = L.b_rows / 4;             // float4 columns of a partial row
-  const int KBper = (a.d / kBK) / split;
-  const int kb0 = rank * KBper, kb1 = kb0 + KBper;
-  const uint32_t ncols = tmem_cols_for(L.b_rows);
+  // Pass split: predict whose weights stream in two passes (N > 128) run by a 2-CTA cluster in
+  // which CTA r streams pass r ([W], then [W_p]) over all of K; the two column halves of every
+  // row then meet in the CTA that finishes it, through distributed shared memory, and are not
+  // summed.  Otherwise the cluster splits K and the S partial rows are summed.
+  const bool psplit = predict && L.passes == 2 && split == 2;
+  const int KBper = psplit ? a.d / kBK : (a.d / kBK) / split;
+  const int kb0 = psplit ? 0 : rank * KBper, kb1 = kb0 + KBper;
+  const int npass = psplit ? 1 : L.passes;  // passes this CTA streams
+  const int pass0 = psplit ? rank : 0;      // the first of them
+  const int acc_cols = psplit ? L.pass_rows : L.b_rows;
+  const uint32_t ncols = tmem_cols_for(acc_cols);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < L.stages; ++s) {
@@ -231,14 +246,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t phase = 0;
       const uint64_t keep = l2_policy_evict_last();    // weights are re-read by every tile
       const uint64_t once = l2_policy_evict_first();   // h is read once
-      for (int kb = kb0; kb < kb1; ++kb) {
+      const int nkb = kb1 - kb0;
+      for (int i = 0; i < npass * nkb; ++i) {
+        const int pass = pass0 + i / nkb;
+        const int kb = kb0 + i % nkb;
         if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, a.status)) break;
         uint8_t* sa = smem + stage * L.stage_bytes;
         uint8_t* sb = sa + kATileBytes;
         mbar_arrive_expect_tx(&full[stage], bytes);
         tma_load_2d_hint(sa, &tm_h, &full[stage], kb * kBK, t0, once);
-        tma_load_2d_hint(sb, &tm_w, &full[stage], kb * kBK, 0, keep);
-        if (predict) tma_load_2d_hint(sb + N * kBK * 2, &tm_wp, &full[stage], kb * kBK, 0, keep);
+        if (L.passes == 1) {
+          tma_load_2d_hint(sb, &tm_w, &full[stage], kb * kBK, 0, keep);
+          if (predict) tma_load_2d_hint(sb + N * kBK * 2, &tm_wp, &full[stage], kb * kBK, 0, keep);
+        } else {
+          tma_load_2d_hint(sb, pass == 0 ? &tm_w : &tm_wp, &full[stage], kb * kBK, 0, keep);
+        }
         issued |= 1u << stage;
         last_par = (last_par & ~(1u << stage)) | (phase << stage);
         if (++stage == L.stages) {
@@ -258,7 +280,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
-      for (int kb = kb0; kb < kb1 && ok; ++kb) {
+      const int nkb = kb1 - kb0;
+      for (int i = 0; i < npass * nkb && ok; ++i) {
+        const int pass = pass0 + i / nkb;
+        const int kb = kb0 + i % nkb;
         if (!mbar_wait(&full[stage], phase, abort_flag, a.status)) {
           ok = false;
           break;
@@ -269,11 +294,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int kk = 0; kk < kBK / 16; ++kk) {
           const uint64_t adesc = umma_desc_sw128(sa + kk * 32);
-          for (int n0 = 0; n0 < L.b_rows; n0 += 256) {
-            const int nc = (L.b_rows - n0) < 256 ? (L.b_rows - n0) : 256;
-            const uint64_t bdesc = umma_desc_sw128(sb + n0 * (kBK * 2) + kk * 32);
-            umma_bf16(tmem + n0, adesc, bdesc, umma_idesc_bf16(kTileM, nc),
-                      (kb > kb0 || kk > 0) ? 1u : 0u);
+          const uint32_t acc = (kb > kb0 || kk > 0) ? 1u : 0u;
+          if (L.passes == 1) {
+            for (int n0 = 0; n0 < L.b_rows; n0 += 256) {
+              const int nc = (L.b_rows - n0) < 256 ? (L.b_rows - n0) : 256;
+              const uint64_t bdesc = umma_desc_sw128(sb + n0 * (kBK * 2) + kk * 32);
+              umma_bf16(tmem + n0, adesc, bdesc, umma_idesc_bf16(kTileM, nc), acc);
+            }
+          } else {  // pass p fills accumulator columns [p N, (p + 1) N): p_old, then b
+            umma_bf16(tmem + (psplit ? 0 : pass * L.pass_rows), adesc,
+                      umma_desc_sw128(sb + kk * 32), umma_idesc_bf16(kTileM, L.pass_rows), acc);
           }
         }
         umma_commit(&empty[stage]);
@@ -369,13 +399,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (split > 1) {
     cluster_sync();  // every CTA has finished its K blocks: the pipeline stages are free
     if (epi && have) {
-      // Reduce-scatter by rows: this TMEM row goes to CTA row / R as its row row % R.
+      // Reduce-scatter by rows: this TMEM row goes to CTA row / R as its row row % R, into the
+      // slot of source `rank` (K split) or into columns [rank N, (rank + 1) N) (pass split).
       float4* recv_w = reinterpret_cast<float4*>(smem);
       const uint32_t dst = static_cast<uint32_t>(row / R);
       const int drow = row - static_cast<int>(dst) * R;
+      const int off4 = psplit ? L.pass_rows / 4 : nb4;
       const uint32_t rbase =
-          mapa_shared(smem_u32(recv_w + (rank * nb4) * R + drow), dst);
-      for (int c0 = 0; c0 < L.b_rows; c0 += 32) {
+          mapa_shared(smem_u32(recv_w + (rank * off4) * R + drow), dst);
+      for (int c0 = 0; c0 < acc_cols; c0 += 32) {
         uint32_t r0[16], r1[16];
         tmem_ld16(trow + c0, r0);
         tmem_ld16(trow + c0 + 16, r1);
@@ -385,7 +417,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int j = 0; j < 4; ++j)
           st_cluster_v4(rbase + static_cast<uint32_t>(((c0 / 4 + j) * R) * 16), r0[4 * j],
                         r0[4 * j + 1], r0[4 * j + 2], r0[4 * j + 3]);
-        if (c0 + 16 < L.b_rows) {  // b_rows is a multiple of 16, not always of 32
+        if (c0 + 16 < acc_cols) {  // a multiple of 16, not always of 32
 #pragma unroll
           for (int j = 0; j < 4; ++j)
             st_cluster_v4(rbase + static_cast<uint32_t>(((c0 / 4 + 4 + j) * R) * 16), r1[4 * j],
@@ -394,7 +426,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     cluster_sync();  // every partial row has landed
-    if (epi) {
+    if (epi && !psplit) {
       // Sum the S received copies of this CTA's rows once, in source order, into source 0's
       // slots: consecutive threads take consecutive 16-byte words (no bank conflicts), so the
       // finishing threads then read one value per column instead of S strided ones.
@@ -872,6 +904,14 @@ int route_split(int T, int N, int d, int mode, int num_sms) {
   const RouteSmemLayout L = route_layout(N, mode == kModePredict, false);
   const int tiles = (T + kTileM - 1) / kTileM;
   const int KB = d / kBK;
+  if (L.passes == 2) {
+    // predict with N > 128: the pass split (two CTAs per tile, each receiving its 64 rows' two
+    // column halves) when it fits in one wave, else one CTA per tile streaming both passes
+    const bool fits = route_recv_bytes(L.b_rows) / 2 <= L.stages * L.stage_bytes &&
+                      KB % 2 == 0 && (N / 2) % 16 == 0 && tiles * 2 <= num_sms &&
+                      max_active_clusters(mode, 2, N) >= tiles;
+    return fits ? 2 : 1;
+  }
   if (route_recv_bytes(L.b_rows) > L.stages * L.stage_bytes) return 1;
   for (int s = kMaxSplit; s > 1; s >>= 1) {
     if (N % s != 0 || (N / s) % 16 != 0 || KB % s != 0 || tiles * s > num_sms) continue;
