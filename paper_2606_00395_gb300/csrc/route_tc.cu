@@ -246,20 +246,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t phase = 0;
       const uint64_t keep = l2_policy_evict_last();    // weights are re-read by every tile
       const uint64_t once = l2_policy_evict_first();   // h is read once
-      const int nkb = kb1 - kb0;
-      for (int i = 0; i < npass * nkb; ++i) {
-        const int pass = pass0 + i / nkb;
-        const int kb = kb0 + i % nkb;
-        if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, a.status)) break;
+      bool ok = true;
+      for (int pass = pass0; pass < pass0 + npass && ok; ++pass)
+      for (int kb = kb0; kb < kb1; ++kb) {
+        if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, a.status)) {
+          ok = false;
+          break;
+        }
         uint8_t* sa = smem + stage * L.stage_bytes;
         uint8_t* sb = sa + kATileBytes;
         mbar_arrive_expect_tx(&full[stage], bytes);
         tma_load_2d_hint(sa, &tm_h, &full[stage], kb * kBK, t0, once);
-        if (L.passes == 1) {
+        if (!predict || L.passes == 1) {  // replay never takes two passes
           tma_load_2d_hint(sb, &tm_w, &full[stage], kb * kBK, 0, keep);
           if (predict) tma_load_2d_hint(sb + N * kBK * 2, &tm_wp, &full[stage], kb * kBK, 0, keep);
+        } else if (pass == 0) {
+          // Each map is named directly: with one pointer selected between the two maps here,
+          // even the replay kernel's mainloop (which never gets here) ran 25 % slower.
+          tma_load_2d_hint(sb, &tm_w, &full[stage], kb * kBK, 0, keep);
         } else {
-          tma_load_2d_hint(sb, pass == 0 ? &tm_w : &tm_wp, &full[stage], kb * kBK, 0, keep);
+          tma_load_2d_hint(sb, &tm_wp, &full[stage], kb * kBK, 0, keep);
         }
         issued |= 1u << stage;
         last_par = (last_par & ~(1u << stage)) | (phase << stage);
@@ -280,10 +286,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
-      const int nkb = kb1 - kb0;
-      for (int i = 0; i < npass * nkb && ok; ++i) {
-        const int pass = pass0 + i / nkb;
-        const int kb = kb0 + i % nkb;
+      for (int pass = pass0; pass < pass0 + npass && ok; ++pass)
+      for (int kb = kb0; kb < kb1 && ok; ++kb) {
         if (!mbar_wait(&full[stage], phase, abort_flag, a.status)) {
           ok = false;
           break;
@@ -295,7 +299,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kk = 0; kk < kBK / 16; ++kk) {
           const uint64_t adesc = umma_desc_sw128(sa + kk * 32);
           const uint32_t acc = (kb > kb0 || kk > 0) ? 1u : 0u;
-          if (L.passes == 1) {
+          if (!predict || L.passes == 1) {  // replay never takes two passes
             for (int n0 = 0; n0 < L.b_rows; n0 += 256) {
               const int nc = (L.b_rows - n0) < 256 ? (L.b_rows - n0) : 256;
               const uint64_t bdesc = umma_desc_sw128(sb + n0 * (kBK * 2) + kk * 32);
