@@ -123,3 +123,23 @@ def make_token_sample(T: int, n: int, seed: int = 0) -> torch.Tensor:
     pick = torch.randperm(T, generator=gen)[: max(n - 2, 0)]
     ids = torch.unique(torch.cat([pick, torch.tensor([0, T - 1])]))
     return ids[:n] if ids.numel() > n else ids
+
+
+def make_loss_inputs(N: int, d: int, Tc: int, T_rho: int, seed: int = 0,
+                     dtype: str = "bf16") -> Dict[str, torch.Tensor]:
+    """Inputs of the predictive loss drawn directly, without a whole layer (for shapes whose
+    expert weights would be needlessly large): cached features h_old [Tc, d] ~ N(0, 1), cached
+    router logits p_old [Tc, N] ~ N(0, 0.5^2), predictor W_pred [N, d] ~ N(0, 0.02^2), a teacher
+    distribution rho [T_rho, N] (u^4 normalised per row, u ~ U(0, 1): skewed but every entry
+    positive) and cache positions pos [Tc] int32 ~ U{0, T_rho - 1}.  Generator seed+4, drawn in
+    that order on the CPU; h_old and W_pred cast once to the layer dtype."""
+    gen = torch.Generator(device="cpu")
+    gen.manual_seed(seed + 4)
+    dt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    h_old = torch.randn(Tc, d, generator=gen).to(dt)
+    p_old = 0.5 * torch.randn(Tc, N, generator=gen)
+    W_pred = (0.02 * torch.randn(N, d, generator=gen)).to(dt)
+    u = torch.rand(T_rho, N, generator=gen, dtype=torch.float64) ** 4
+    rho = (u / u.sum(dim=1, keepdim=True)).float()
+    pos = torch.randint(0, T_rho, (Tc,), generator=gen, dtype=torch.int64).to(torch.int32)
+    return dict(h_old=h_old, p_old=p_old, W_pred=W_pred, rho=rho, pos=pos)

@@ -88,6 +88,25 @@ def test_predictor_loss_matches_oracle(name, delta):
     _check(cfg, c, g, delta=delta)
 
 
+# Gradient-GEMM splits the layer cases above do not reach (inputs drawn directly): 8 CTAs per
+# cluster (two 128 x 128 tiles, 8 K blocks), and one CTA per tile (N = 256, d = 4864: 76 tiles,
+# too many for 2-CTA clusters to be resident at once)
+DIRECT = {
+    "split8": (64, 256, 512, 700),
+    "split1_many_tiles": (256, 4864, 192, 300),
+}
+
+
+@pytest.mark.parametrize("name", list(DIRECT))
+def test_predictor_loss_gradient_splits(name):
+    N, d, Tc, T_rho = DIRECT[name]
+    cfg = synth.LayerConfig(name, T=T_rho, d=d, N=N, k=8, m=128)
+    c = synth.make_loss_inputs(N, d, Tc, T_rho, seed=11)
+    c["pos"] = c["pos"].numpy()
+    g = _gpu(cfg, c)
+    _check(cfg, c, g)
+
+
 def test_predictor_loss_full_cache_of_the_qwen3_layer():
     """T = 4096 tokens, T_c = 2048 cached (Table 4's Qwen3 cache length): the loss, every
     per-token KL and the whole gradient."""
