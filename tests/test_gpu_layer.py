@@ -314,6 +314,44 @@ def test_replay_layer_call_equals_the_two_calls(name):
     assert (want_status & B.PR2_STATUS_BAD_INDEX) == (B.PR2_STATUS_BAD_INDEX if cfg.T > 3 else 0)
 
 
+def test_replay_layer_call_in_a_cuda_graph():
+    """The replay layer captured into a CUDA graph on a side stream: replaying the graph on new
+    inputs gives bit for bit what the eager call gives (the routing kernel launched behind the
+    expert GEMMs, with its late dependency wait, is captured like the rest)."""
+    cfg = SMALL["bf16_multitile"]
+    L = synth.make_layer(cfg, seed=13)
+    Ld = H.to_dev(L)
+    W2 = synth.make_drifted_router(L["W_router"], seed=13).cuda()
+    g = H.gpu_predict(cfg, Ld)
+    dm = H.dims_of(cfg)
+    ws = B.alloc_workspace(dm)
+    x = Ld["x"].clone()
+    gates = torch.empty(cfg.T, cfg.k, dtype=torch.float32, device="cuda")
+    probs = torch.empty(cfg.T, cfg.N, dtype=torch.float32, device="cuda")
+    out = torch.empty_like(x)
+
+    def layer(stream=None):
+        return B.pr2_moe_replay_forward(dm, x, W2, g["idx"], gates, probs, Ld["W_gate"],
+                                        Ld["W_up"], Ld["W_down"], None, None, None, out,
+                                        workspace=ws, stream=stream)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        assert layer(side) == 0  # warm-up outside the capture
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=side):
+        assert layer(side) == 0
+    x.copy_(torch.roll(Ld["x"], 1, 0))  # new inputs for the replay
+    graph.replay()
+    torch.cuda.synchronize()
+    got = (gates.clone(), probs.clone(), out.clone())
+    assert layer() == 0
+    torch.cuda.synchronize()
+    assert torch.equal(got[0], gates) and torch.equal(got[1], probs) and torch.equal(got[2], out)
+
+
 @pytest.mark.parametrize("name", ["tiny_fp32", "bf16_fused_dispatch", "bf16_multitile",
                                   "bf16_partial_n", "bf16_shared_n256", "bf16_top1",
                                   "bf16_one_token"])
