@@ -161,6 +161,25 @@ def test_near_tie_counter_tracks_the_oracle_margin():
     assert abs(n_gpu - n_orc) <= borderline, (n_gpu, n_orc, borderline)
 
 
+@pytest.mark.parametrize("d", [192, 256])
+def test_predict_routing_with_256_experts_in_two_passes(d):
+    """N = 256: the router and predictor weights stream in two passes over K.  d = 256 (an even
+    number of K blocks) runs them as the pass split, one pass per CTA of a 2-CTA cluster whose
+    column halves meet unsummed; d = 192 (three K blocks) runs both passes in one CTA.  Routes
+    under the near-tie rule, gates and p_old logits against the oracle; T = 300 leaves a ragged
+    last tile."""
+    cfg = synth.LayerConfig("p256", T=300, d=d, N=256, k=8, m=128)
+    L = synth.make_layer(cfg, seed=d)
+    Ld = H.to_dev(L)
+    g = H.gpu_predict(cfg, Ld)
+    assert int(g["status"].item()) == 0
+    orc = oracle.route_predict(L["x"], L["W_router"], L["W_pred"], cfg.k)
+    idx = H.cpu(g["idx"]).numpy()
+    H.check_routes(orc, idx)
+    H.rowwise_close(H.cpu(g["gates"]).numpy(), np.take_along_axis(orc["probs"], idx, 1))
+    H.rowwise_close(H.cpu(g["logits"]).numpy(), orc["logits"])
+
+
 def test_zero_predictor_replay_reproduces_rollout():
     """W_p = 0 and the same router: replaying the recorded route gives the rollout gates and
     the same layer output (routing replay, R2, is Pr^2 with a zero predictor)."""
