@@ -193,6 +193,62 @@ def test_rollout_layers_rejects_bad_arguments(lib):
     assert lib.pr2_rollout_layers(*sync, fake, ctypes.c_size_t(ws), None, None) == 1
 
 
+def test_one_call_layers_reject_bad_arguments_on_the_host(lib):
+    """pr2_moe_rollout_forward / pr2_moe_replay_forward check everything both of their steps
+    need before launching anything (these are not device buffers: nothing may be touched)."""
+    fake, odd = ctypes.c_void_p(256), ctypes.c_void_p(258)
+    dm = B.dims(64, 2048, 128, 8, 768)
+    ws = ctypes.c_size_t(B.pr2_moe_workspace_bytes(dm))
+    tail = [None, None, fake, ws, None, None, None]  # counts, perm, workspace, ws_bytes, status, events, stream
+    # rollout: dims, h, W_router, W_pred, idx, gates, logits_old, near_tie, W_gate, W_up, W_down,
+    # Ws_gate, Ws_up, Ws_down, out, ...
+    roll = [ctypes.byref(dm), fake, fake, fake, fake, fake, None, None, fake, fake, fake, None,
+            None, None, fake]
+
+    def rollout(**edit):
+        a = list(roll)
+        t = list(tail)
+        for i, v in edit.get("a", {}).items():
+            a[i] = v
+        for i, v in edit.get("t", {}).items():
+            t[i] = v
+        return lib.pr2_moe_rollout_forward(*a, *t)
+    assert rollout(a={2: None}) == 1             # no router
+    assert rollout(a={3: None}) == 1             # no predictor
+    assert rollout(a={3: odd}) == 1              # misaligned predictor
+    assert rollout(a={6: odd}) == 1              # misaligned logits_old
+    assert rollout(a={1: None}) == 1             # no h (checked for the forward step)
+    assert rollout(a={11: fake}) == 1            # shared weights without shared experts
+    assert rollout(t={3: ctypes.c_size_t(ws.value - 1)}) == 6  # short workspace
+    dms = B.dims(64, 2048, 128, 8, 768, flags=B.PR2_F_SYNC_STATUS)
+    assert rollout(a={0: ctypes.byref(dms)}) == 1  # sync-status needs a status word
+    # replay: dims, h, W_router, idx, gates, probs, W_gate, W_up, W_down, Ws_gate, Ws_up,
+    # Ws_down, out, ...
+    rep = [ctypes.byref(dm), fake, fake, fake, fake, None, fake, fake, fake, None, None, None,
+           fake]
+
+    def replay(**edit):
+        a = list(rep)
+        t = list(tail)
+        for i, v in edit.get("a", {}).items():
+            a[i] = v
+        for i, v in edit.get("t", {}).items():
+            t[i] = v
+        return lib.pr2_moe_replay_forward(*a, *t)
+    assert replay(a={2: None}) == 1              # no router
+    assert replay(a={2: odd}) == 1               # misaligned router
+    assert replay(a={4: None}) == 1              # no gates to write
+    assert replay(a={5: odd}) == 1               # misaligned probs
+    assert replay(a={3: None}) == 1              # no route
+    assert replay(t={2: None}) == 6              # no workspace
+    # an empty layer is a no-op for both, whatever the pointers
+    d0 = B.dims(0, 2048, 128, 8, 768)
+    assert lib.pr2_moe_rollout_forward(ctypes.byref(d0), *([None] * 17), ctypes.c_size_t(0),
+                                       None, None, None) == 0
+    assert lib.pr2_moe_replay_forward(ctypes.byref(d0), *([None] * 15), ctypes.c_size_t(0),
+                                      None, None, None) == 0
+
+
 def test_unknown_flags_are_rejected(lib):
     ok = B.dims(64, 2048, 128, 8, 768, flags=B.PR2_F_NORMALIZE_TOPK | B.PR2_F_SYNC_STATUS)
     assert B.pr2_moe_workspace_bytes(ok) > 0
