@@ -247,7 +247,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
-    if (kKind != kExpertGateUpGather) tma_prefetch_desc(&tm_a);
+    tma_prefetch_desc(&tm_a);
     if (kHas0) {
       tma_prefetch_desc(&tm_b0);
       tma_prefetch_desc(&tm_b1);
@@ -462,7 +462,7 @@ cudaError_t launch_expert_tc(ExpertKind kind, const CUtensorMap& tm_a, const CUt
   const bool has0 = kind != kExpertDown, has1 = kind == kExpertDown || kind == kExpertFused;
   const GemmArgs& gs = has0 ? a.p[0] : a.p[1];
   if (gs.max_tiles <= 0) return cudaSuccess;
-  if ((kind == kExpertGateUpGather || kind == kExpertFused) &&
+  if (kind == kExpertFused &&
       (a.p[0].a_src == nullptr || a.p[0].perm == nullptr || a.p[0].k <= 0))
     return cudaErrorInvalidValue;
   if (kind == kExpertFused && a.ready == nullptr) return cudaErrorInvalidValue;
@@ -472,10 +472,9 @@ cudaError_t launch_expert_tc(ExpertKind kind, const CUtensorMap& tm_a, const CUt
   const int64_t bound = static_cast<int64_t>(gs.max_tiles) * per_tile;
   const int grid = static_cast<int>(bound < num_sms ? bound : num_sms);
   void (*kernel)(CUtensorMap, CUtensorMap, CUtensorMap, CUtensorMap, MlpArgs) =
-      kind == kExpertGateUpGather ? expert_tc_kernel<kExpertGateUpGather>
-      : kind == kExpertGateUpTma  ? expert_tc_kernel<kExpertGateUpTma>
-      : kind == kExpertDown       ? expert_tc_kernel<kExpertDown>
-                                  : expert_tc_kernel<kExpertFused>;
+      kind == kExpertGateUpTma ? expert_tc_kernel<kExpertGateUpTma>
+      : kind == kExpertDown    ? expert_tc_kernel<kExpertDown>
+                               : expert_tc_kernel<kExpertFused>;
   cudaError_t err =
       cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   if (err != cudaSuccess) return err;

@@ -160,11 +160,11 @@ struct GemmArgs {
 // Launch kinds of the tcgen05 grouped GEMM (expert_tc.cu).  Phase 0 is a gate/up GEMM with the
 // SwiGLU epilogue (weights tm_b0 = gate, tm_b1 = up), phase 1 a down GEMM (weights tm_b2).
 enum ExpertKind : int {
-  kExpertGateUpGather = 0,  // phase 0, A rows gathered from p[0].a_src through p[0].perm
   kExpertGateUpTma = 1,     // phase 0, A rows from tm_a (shared experts: rows of h)
   kExpertDown = 2,          // phase 1, A rows from tm_a
-  kExpertFused = 3,         // phase 0 (gathered) then phase 1 (A = p[0].out through tm_a) in
-                            // one cooperative launch
+  kExpertFused = 3,         // phase 0, A rows gathered from p[0].a_src through p[0].perm,
+                            // then phase 1 (A = p[0].out through tm_a), in one cooperative
+                            // launch (the routed experts)
 };
 struct MlpArgs {
   GemmArgs p[2];     // arguments of phase 0 and phase 1 (only the launched phases are read)
