@@ -145,13 +145,7 @@ __device__ __forceinline__ void tma_load_2d_hint(void* smem_dst, const void* tma
 // written through the generic proxy: the thread that acquires the barrier executes
 // fence.proxy.async before a tcgen05.mma (async proxy) reads it.
 // ------------------------------------------------------------------------------------------
-__device__ __forceinline__ void cp_async_16(uint32_t smem_dst, const void* src,
-                                            uint32_t src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_dst), "l"(src),
-               "r"(src_bytes)
-               : "memory");
-}
-// Same with an L2 eviction-priority hint (a createpolicy value).
+// With an L2 eviction-priority hint (a createpolicy value).
 __device__ __forceinline__ void cp_async_16_hint(uint32_t smem_dst, const void* src,
                                                  uint32_t src_bytes, uint64_t policy) {
   asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2, %3;" ::"r"(smem_dst),
@@ -358,10 +352,6 @@ __device__ __forceinline__ void st_cluster_v4(uint32_t addr, uint32_t a, uint32_
                                               uint32_t d) {
   asm volatile("st.shared::cluster.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b),
                "r"(c), "r"(d)
-               : "memory");
-}
-__device__ __forceinline__ void st_cluster_v2(uint32_t addr, uint32_t a, uint32_t b) {
-  asm volatile("st.shared::cluster.v2.b32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b)
                : "memory");
 }
 
